@@ -1,0 +1,463 @@
+"""Benchmark: streaming chunk-causal attention on the 1080p-shaped workload.
+
+One step streams a whole synthetic 1080p-shaped video through the library:
+15 chunks of 2 latent frames x 8160 tokens, 12 heads, d = 128, each chunk one
+KV-cache append plus one chunk-causal attention forward over every earlier
+chunk (Sec. 3.1 with an unbounded window).  The metric is attention TFLOP/s
+counted on visible (query, key) pairs only, 4*B*H*Lq*Lk*d per chunk.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Under torchrun (N > 1) every rank streams its own video (weak scaling: the
+videos are independent units, no data-path collective); the timed region is
+bracketed by a barrier and CUDA synchronisation and the max over ranks is
+reported.  `--impl reference` times the CPU oracle on this host's cores on a
+bounded sample of the same workload (no GPU work).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+HOST_CORES = len(os.sched_getaffinity(0))
+os.environ.setdefault("OPENBLAS_NUM_THREADS", str(HOST_CORES))
+os.environ.setdefault("OMP_NUM_THREADS", str(HOST_CORES))
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2609_36757_gb300 import workloads as WL  # noqa: E402
+
+METRIC = "chunk-causal attn TFLOP/s and % of GB300 bf16 peak; ms per 1080p chunk"
+UNIT = "TFLOP/s"
+WORKLOAD = WL.W1080P
+
+
+def chunk_flops(w: WL.Workload, visible_tokens: int, c: int) -> float:
+    """QK^T plus PV over visible pairs: 4 * B * H * Lq * Lk * d."""
+    lq = w.frames_in_chunk(c) * w.tokens_per_frame
+    return 4.0 * w.batch * w.heads * lq * visible_tokens * w.head_dim
+
+
+def visible_tokens_per_chunk(w: WL.Workload):
+    """Lk of each chunk from the library's own visibility plan (host only)."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    cfg = FV.config_from_workload(w)
+    plan = FV.fastvr_attn_plan(cfg, 1 << 40, FV.fastvr_kv_cache_bytes(cfg))
+    out = []
+    try:
+        for c in range(w.num_chunks):
+            FV.fastvr_plan_set_state(plan, c + 1, w.frames_in_chunk(c))
+            out.append(FV.fastvr_plan_visible(plan)[1])
+    finally:
+        FV.fastvr_plan_destroy(plan)
+    return out
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
+            "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def load_traffic(kernel: str):
+    """DRAM bytes per launch from a committed ncu summary, when that summary
+    was taken on the current kernel source (else None)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    kv = {}
+    for line in open(path):
+        if "=" in line and not line.startswith("#"):
+            k, v = line.strip().split("=", 1)
+            kv[k.strip()] = v.strip()
+    src = os.path.join(ROOT, "paper_2609_36757_gb300", "csrc", kv.get("source", ""))
+    if not os.path.exists(src):
+        return None
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    if digest != kv.get("source_sha256_16"):
+        return None
+    return float(kv["dram_bytes_per_avg_launch"])
+
+
+# ------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.device_index = device_index
+
+    def start(self):
+        try:
+            ident = str(self.device_index)
+            try:
+                ident = "GPU-" + str(torch.cuda.get_device_properties(
+                    self.device_index).uuid)
+            except Exception:
+                pass
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", ident, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            return None
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for n, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------- CPU oracle
+class OracleSample:
+    """The oracle timed on the last chunk of a workload (its largest visible
+    window), head 0 of batch 0, in blocks of query rows."""
+
+    def __init__(self, w: WL.Workload, chunks, rows_per_block: int = 256):
+        from oracle import attention as OA
+        self.OA, self.w, self.rows = OA, w, rows_per_block
+        self.c = len(chunks) - 1
+        vis = OA.visible_chunks(self.c, w.window_chunks)
+        self.k = np.concatenate([chunks[j][1][0, :, 0].float().numpy()
+                                 for j in vis]).astype(np.float64)
+        self.v = np.concatenate([chunks[j][2][0, :, 0].float().numpy()
+                                 for j in vis]).astype(np.float64)
+        self.q = chunks[self.c][0][0, :, 0].float().numpy().astype(np.float64)
+        self.next_row = 0
+
+    def run(self, seconds: float, max_blocks: int):
+        """Returns (TFLOP/s, description)."""
+        lk = self.k.shape[0]
+        flops, blocks = 0.0, 0
+        t0 = time.perf_counter()
+        while blocks < max_blocks:
+            r0 = self.next_row
+            qb = self.q[r0:r0 + self.rows]
+            self.next_row = (r0 + self.rows) % self.q.shape[0]
+            self.OA.softmax_attention(qb, self.k, self.v, self.w.softmax_scale)
+            flops += 4.0 * qb.shape[0] * lk * self.w.head_dim
+            blocks += 1
+            if time.perf_counter() - t0 >= seconds:
+                break
+        dt = time.perf_counter() - t0
+        desc = (f"oracle fp64 (numpy) on chunk {self.c} of {self.w.name}: "
+                f"{blocks} block(s) of {self.rows} query rows x Lk={lk} keys, "
+                f"head 0, {dt:.2f} s")
+        return flops / dt / 1e12, desc
+
+
+def host_chunks(w: WL.Workload, seed_offset: int = 0):
+    if seed_offset:
+        import dataclasses
+        w = dataclasses.replace(w, seed=w.seed + seed_offset)
+    return [(q, k, v) for _, q, k, v in WL.chunk_stream(w)]
+
+
+# ------------------------------------------------------------- arms
+def run_reference(args, rank: int, world: int) -> None:
+    if rank != 0:
+        return
+    w = WORKLOAD
+    sample = OracleSample(w, host_chunks(w))
+    for _ in range(args.warmup):
+        sample.run(0.0, 1)
+    vals = []
+    for _ in range(args.steps):
+        v, desc = sample.run(0.0, 1)
+        vals.append(v)
+    value = statistics.median(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic (seeded N(0,1) bf16 inputs)",
+        "config": {"workload": w.name, "batch": w.batch, "heads": w.heads,
+                   "head_dim": w.head_dim, "tokens_per_frame": w.tokens_per_frame,
+                   "frames_per_chunk": w.frames_per_chunk,
+                   "chunks": w.num_chunks, "window_chunks": w.window_chunks},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": HOST_CORES,
+                         "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
+    from paper_2609_36757_gb300 import fastvr as FV
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = WORKLOAD
+    lk = visible_tokens_per_chunk(w)
+    flops = [chunk_flops(w, lk[c], c) for c in range(w.num_chunks)]
+    step_flops = sum(flops)
+
+    chunks = host_chunks(w, seed_offset=rank)
+    dq = [q.to(dev) for q, _, _ in chunks]
+    dk = [k.to(dev) for _, k, _ in chunks]
+    dv = [v.to(dev) for _, _, v in chunks]
+    douts = [torch.empty_like(q) for q in dq]
+    att = FV.StreamingAttention(FV.config_from_workload(w), dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        att.reset()
+        for c in range(w.num_chunks):
+            if ev is not None:
+                ev[c][0].record(stream)
+            att.append(dk[c], dv[c])
+            if ev is not None:
+                ev[c][1].record(stream)
+            att.forward(dq[c], out=douts[c])
+            if ev is not None:
+                ev[c][2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    if att.status() != FV.FASTVR_OK:
+        raise RuntimeError("device-side failure during warm-up")
+
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            for _ in range(w.num_chunks)] for _ in range(args.steps)]
+    clocks = ClockSampler(local_rank) if rank == 0 else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for s in range(args.steps):
+        step(evs[s])
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clock_info = clocks.stop() if clocks else None
+    elapsed_ms = t_start.elapsed_time(t_end)
+    if att.status() != FV.FASTVR_OK:
+        raise RuntimeError("device-side failure in the timed region")
+
+    fwd_ms = [[evs[s][c][1].elapsed_time(evs[s][c][2]) for c in range(w.num_chunks)]
+              for s in range(args.steps)]
+    app_ms = [[evs[s][c][0].elapsed_time(evs[s][c][1]) for c in range(w.num_chunks)]
+              for s in range(args.steps)]
+    max_ms = reduce_max(elapsed_ms, world)
+    value = world * step_flops * args.steps / (max_ms / 1e3) / 1e12
+
+    e2e = (None if args.skip_e2e else
+           run_e2e(args, w, chunks, att, dev, step_flops, world))
+
+    if rank != 0:
+        return
+    peaks, peak_kind = load_peaks()
+    fwd_total_ms = sum(map(sum, fwd_ms))
+    attn_tflops = step_flops * args.steps / (fwd_total_ms / 1e3) / 1e12
+    app_total_ms = sum(map(sum, app_ms))
+    app_bytes = sum(2 * 2 * w.batch * w.heads * w.frames_in_chunk(c) *
+                    w.tokens_per_frame * w.head_dim for c in range(w.num_chunks))
+    app_gbs = app_bytes * args.steps / (app_total_ms / 1e3) / 1e9
+    per_chunk_fwd = [statistics.median(fwd_ms[s][c] for s in range(args.steps))
+                     for c in range(w.num_chunks)]
+    peak = peaks["bf16_tflops_sustained"]
+    traffic = load_traffic("chunk_attn_fwd_1080p")
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": max_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V, one video per GPU)",
+        "config": {"workload": w.name, "batch": w.batch, "heads": w.heads,
+                   "head_dim": w.head_dim, "tokens_per_frame": w.tokens_per_frame,
+                   "frames_per_chunk": w.frames_per_chunk,
+                   "chunks": w.num_chunks, "window_chunks": w.window_chunks,
+                   "step": "reset + 15 x (kv_append + chunk_attn_fwd)",
+                   "l2": "inputs larger than L2 (visible K/V per chunk "
+                         "0.1-1.5 GB, 2.3 GB of Q/K/V per step)",
+                   "parallelism": f"replicas x{world} (one video per GPU)"},
+        "ms_per_chunk": {"mean_fwd": statistics.mean(per_chunk_fwd),
+                         "last_fwd": per_chunk_fwd[-1],
+                         "mean_append": app_total_ms / args.steps / w.num_chunks},
+        "latent_frames_per_s": world * w.num_frames * args.steps / (max_ms / 1e3),
+        "attn_kernel_tflops": attn_tflops,
+        "frac_of_burst_peak": attn_tflops / peaks["bf16_tflops"],
+        "append_gbs": app_gbs,
+        "append_frac_of_hbm": app_gbs / peaks["hbm_gbs"],
+        "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peak,
+                     "unit": "TFLOP/s", "frac": attn_tflops / peak,
+                     "peak_kind": f"{peak_kind} bf16 sustained",
+                     "kernel": "chunk_attn_fwd",
+                     "traffic": traffic},
+        "gpu_launches": 2 * w.num_chunks * args.steps,
+        "clocks": clock_info,
+        "e2e": e2e,
+    }
+    if world == 1 and args.cpu_seconds > 0:
+        cpu_v, desc = OracleSample(w, chunks).run(args.cpu_seconds, 10 ** 6)
+        line["cpu_baseline"] = {"value": cpu_v, "unit": UNIT,
+                                "cores": HOST_CORES, "kind": "oracle",
+                                "sample": desc}
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, w, chunks, att, dev, step_flops, world):
+    """The same metric through the public API from pinned host buffers: every
+    step copies each chunk's Q/K/V host->device (a side stream, overlapped
+    with the previous chunk's compute) and each output device->host."""
+    pq = [q.pin_memory() for q, _, _ in chunks]
+    pk = [k.pin_memory() for _, k, _ in chunks]
+    pv = [v.pin_memory() for _, _, v in chunks]
+    po = [torch.empty_like(q).pin_memory() for q in pq]
+    slots = [[torch.empty_like(pq[0], device=dev) for _ in range(3)]
+             for _ in range(2)]
+    outs = [torch.empty_like(pq[0], device=dev) for _ in range(2)]
+    compute = torch.cuda.current_stream(dev)
+    h2d = torch.cuda.Stream(dev)
+    d2h = torch.cuda.Stream(dev)
+    h2d_bytes = sum(t.numel() * 2 for t in pq + pk + pv)
+    d2h_bytes = sum(t.numel() * 2 for t in po)
+
+    def step():
+        att.reset()
+        free = [torch.cuda.Event(), torch.cuda.Event()]
+        out_free = [torch.cuda.Event(), torch.cuda.Event()]
+        for e in free + out_free:
+            e.record(compute)
+        for c in range(w.num_chunks):
+            s = c % 2
+            L = pq[c].shape[1]
+            sq, sk, sv = (x[:, :L] for x in slots[s])
+            with torch.cuda.stream(h2d):
+                h2d.wait_event(free[s])
+                sq.copy_(pq[c], non_blocking=True)
+                sk.copy_(pk[c], non_blocking=True)
+                sv.copy_(pv[c], non_blocking=True)
+                ready = torch.cuda.Event()
+                ready.record(h2d)
+            compute.wait_event(ready)
+            compute.wait_event(out_free[s])
+            att.append(sk, sv)
+            o = outs[s][:, :L]
+            att.forward(sq, out=o)
+            free[s].record(compute)
+            done = torch.cuda.Event()
+            done.record(compute)
+            with torch.cuda.stream(d2h):
+                d2h.wait_event(done)
+                po[c].copy_(o, non_blocking=True)
+                out_free[s].record(d2h)
+        compute.wait_stream(d2h)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    dt = reduce_max(time.perf_counter() - t0, world)
+    return {"value": world * step_flops * args.steps / dt / 1e12, "unit": UNIT,
+            "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h_bytes}
+
+
+# ------------------------------------------------------------- distributed
+def barrier(world: int) -> None:
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def reduce_max(x: float, world: int) -> float:
+    if world <= 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="fastvr", choices=["fastvr", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="CPU-baseline sample length (0 skips it)")
+    ap.add_argument("--chunks", type=int, default=0,
+                    help="stream only the first N chunks (small profiling "
+                         "cases); 0 = the whole workload")
+    ap.add_argument("--skip-e2e", action="store_true",
+                    help="omit the end-to-end leg (profiling cases)")
+    args = ap.parse_args(argv)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    global WORKLOAD
+    if args.chunks:
+        import dataclasses
+        WORKLOAD = dataclasses.replace(WORKLOAD, num_chunks=args.chunks,
+                                       name=f"{WORKLOAD.name}-first{args.chunks}")
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_gpu(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,162 @@
+/*
+ * fastvr_attn.h -- C ABI of the GB300 (sm_103a) chunk-wise causal attention
+ * library for streaming video diffusion transformers.
+ *
+ * The operation (FastVR, Sec. 3.1 "Chunk-wise causal attention", Eq. 1):
+ * latent frames are grouped into non-overlapping chunks of k frames; a query
+ * of frame i sees a key of frame j iff floor(i/k) - floor(j/k) lies in
+ * {0, ..., W}.  Eq. 1 itself is W = 1; window_chunks = -1 widens the set to
+ * every earlier chunk.  Inference processes the chunks one after the other
+ * and keeps the keys and values of the chunks that later queries still see in
+ * a KV cache (Sec. 3.1, last paragraph), so a chunk's cost is bounded by its
+ * visible window and the cache holds O(k) tokens for a bounded window.
+ *
+ * Per chunk c, in stream order:
+ *   fastvr_kv_append(plan, K_c, V_c, f_c, stream);        // K/V into the cache
+ *   fastvr_chunk_attn_fwd(plan, Q_c, O_c, lse_c, stream);  // Q_c over its window
+ *
+ * Conventions shared by every entry point:
+ *  - The caller owns all device memory (cache, q, k, v, out, lse).  The plan
+ *    owns host state only and binds the cache pointer given at plan time.
+ *  - Tensors are bfloat16, contiguous, 16-byte aligned.  Per-chunk tensors are
+ *    token-major [B, f*N, H, d] (the layout a fused QKV projection emits);
+ *    out has the same layout; lse is float32 [B, H, f*N] (natural log).
+ *  - Device pointers are CUDA device addresses on the current device; the
+ *    stream argument is a cudaStream_t (NULL = legacy default stream).  Work
+ *    is enqueued on that stream; nothing is synchronised by the library except
+ *    in fastvr_get_status.
+ *  - Errors are returned as status codes; nothing throws or aborts across the
+ *    ABI.  A call that returns an error enqueues no work and leaves the plan's
+ *    counters unchanged.  Device-side failures (a bounded wait that gave up)
+ *    are recorded in the cache's control word and reported by
+ *    fastvr_get_status.
+ *  - There is no CPU fallback: on a device that is not sm_103 the first
+ *    device call returns FASTVR_ERR_UNSUPPORTED.
+ *  - A plan is not thread-safe; use one plan per stream of chunks.
+ */
+#ifndef FASTVR_ATTN_H_
+#define FASTVR_ATTN_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define FASTVR_API __attribute__((visibility("default")))
+#else
+#define FASTVR_API
+#endif
+
+struct CUstream_st; /* cudaStream_t is struct CUstream_st* */
+
+typedef enum {
+  FASTVR_OK = 0,
+  FASTVR_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, bad shape, frames<1 */
+  FASTVR_ERR_UNSUPPORTED = 2,  /* head_dim not 64/128, device not sm_103      */
+  FASTVR_ERR_CAPACITY = 3,     /* frames > k, more chunks than max_chunks,
+                                  cache buffer too small                      */
+  FASTVR_ERR_SEQUENCE = 4,     /* fwd before any append; append after a
+                                  ragged (final) chunk                        */
+  FASTVR_ERR_CUDA = 5,         /* a CUDA runtime/driver call failed           */
+  FASTVR_ERR_TIMEOUT = 6       /* a bounded device-side wait gave up          */
+} fastvr_status_t;
+
+typedef struct {
+  int32_t batch;             /* B: videos or spatial tiles                    */
+  int32_t heads;             /* H                                             */
+  int32_t head_dim;          /* d: 64 or 128                                  */
+  int32_t tokens_per_frame;  /* N: tokens of one latent frame                 */
+  int32_t frames_per_chunk;  /* k: latent frames per chunk (Eq. 1)            */
+  int32_t window_chunks;     /* W: earlier chunks a chunk sees; Eq. 1 is 1;
+                                -1 = every earlier chunk                      */
+  int32_t max_chunks;        /* capacity in chunks when window_chunks == -1;
+                                ignored otherwise                             */
+  float softmax_scale;       /* 0 => 1/sqrt(head_dim)                         */
+} fastvr_attn_config_t;
+
+typedef struct fastvr_plan_s* fastvr_plan_t;
+
+/* Bytes of device memory the caller must provide for the KV cache of cfg:
+ * K and V, each [B, H, S*k*N, d] bfloat16 with S = window_chunks + 1 slots
+ * (bounded window) or max_chunks slots (unbounded), plus a 256-byte control
+ * block at the end.  Host only; no device work.
+ * Errors: INVALID_ARG (null, non-positive sizes), UNSUPPORTED (head_dim). */
+FASTVR_API fastvr_status_t fastvr_kv_cache_bytes(const fastvr_attn_config_t* cfg,
+                                      size_t* bytes);
+
+/* Validate cfg and bind a caller-owned cache buffer of `bytes` bytes (device
+ * memory, 256-byte aligned, at least fastvr_kv_cache_bytes).  The cache
+ * contents need no initialisation.  Host only: device set-up (TMA
+ * descriptors, device check, clearing the control block) happens on the
+ * first device call.  *out receives a new plan, released by
+ * fastvr_plan_destroy.
+ * Errors: INVALID_ARG, UNSUPPORTED, CAPACITY (buffer too small). */
+FASTVR_API fastvr_status_t fastvr_attn_plan(const fastvr_attn_config_t* cfg,
+                                 void* kv_cache, size_t bytes,
+                                 fastvr_plan_t* out);
+
+/* KV caching for streaming inference (Sec. 3.1): copy the next chunk's keys
+ * and values, k_new and v_new bfloat16 [B, frames*N, H, d] token-major, into
+ * cache slot (c mod S) at token offset (c mod S)*k*N of the head-major cache,
+ * where c is the plan's chunk counter, then advance the counter.  The copy is
+ * bit-exact.  frames is 1..k; frames < k marks the final (ragged) chunk of the
+ * stream, after which appends fail until fastvr_plan_reset.
+ * Errors: INVALID_ARG, CAPACITY (frames > k; unbounded window and c ==
+ * max_chunks), SEQUENCE (after a ragged chunk), UNSUPPORTED, CUDA. */
+FASTVR_API fastvr_status_t fastvr_kv_append(fastvr_plan_t plan, const void* k_new,
+                                 const void* v_new, int32_t frames,
+                                 struct CUstream_st* stream);
+
+/* Chunk-causal attention of the most recently appended chunk c (Eq. 1 with
+ * window W): q bfloat16 [B, f_c*N, H, d] token-major attends to the cached
+ * keys/values of chunks max(0, c-W) .. c (all of 0..c when unbounded), with
+ * softmax scale cfg.softmax_scale, accumulating in float32.  out receives
+ * bfloat16 [B, f_c*N, H, d]; lse (nullable) receives float32 [B, H, f_c*N],
+ * the natural-log sum of exp(scaled scores).  Only visible cache slots are
+ * read.  Does not advance the chunk counter (may be repeated).
+ * Errors: INVALID_ARG, SEQUENCE (no chunk appended yet), UNSUPPORTED, CUDA. */
+FASTVR_API fastvr_status_t fastvr_chunk_attn_fwd(fastvr_plan_t plan, const void* q,
+                                      void* out, float* lse,
+                                      struct CUstream_st* stream);
+
+/* Start a new video: chunk counter back to 0; the cache contents are ignored
+ * from then on.  Host only. */
+FASTVR_API fastvr_status_t fastvr_plan_reset(fastvr_plan_t plan);
+
+/* Synchronise the device, then report (and clear) any device-side failure
+ * recorded in the cache's control block: FASTVR_ERR_TIMEOUT when a bounded
+ * wait inside a kernel gave up, FASTVR_ERR_CUDA when a CUDA error is pending,
+ * FASTVR_OK otherwise. */
+FASTVR_API fastvr_status_t fastvr_get_status(fastvr_plan_t plan);
+
+/* Streaming state for checkpoint/resume: the number of chunks appended and
+ * the frame count of the newest chunk.  Together with the cache bytes it is
+ * the whole state of a stream.  Host only. */
+FASTVR_API fastvr_status_t fastvr_plan_get_state(fastvr_plan_t plan, int64_t* chunks,
+                                      int32_t* last_frames);
+FASTVR_API fastvr_status_t fastvr_plan_set_state(fastvr_plan_t plan, int64_t chunks,
+                                      int32_t last_frames);
+
+/* The visible key set of the most recently appended chunk as at most two
+ * contiguous token ranges of one head's cache [start, start+len) (the ring
+ * wraps), and their total Lk.  This is the set fastvr_chunk_attn_fwd reads.
+ * seg_start and seg_len must hold 2 entries.  Host only.
+ * Errors: INVALID_ARG, SEQUENCE (no chunk appended). */
+FASTVR_API fastvr_status_t fastvr_plan_visible(fastvr_plan_t plan, int32_t* num_segments,
+                                    int64_t* seg_start, int64_t* seg_len,
+                                    int64_t* visible_tokens);
+
+/* Release a plan (host memory only; the cache stays the caller's). */
+FASTVR_API void fastvr_plan_destroy(fastvr_plan_t plan);
+
+/* A static, human-readable name for a status code. */
+FASTVR_API const char* fastvr_status_string(fastvr_status_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FASTVR_ATTN_H_ */

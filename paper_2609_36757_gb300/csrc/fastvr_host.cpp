@@ -1,0 +1,325 @@
+// Host side of the chunk-causal attention library: the C ABI declared in
+// include/fastvr_attn.h.  Plans, ring-slot bookkeeping and the visibility
+// computation are plain host code; the device work is in kv_append.cu and
+// chunk_attn_fwd.cu.
+//
+// Visibility (Sec. 3.1, Eq. 1, window W): chunk c's queries see the keys of
+// chunks max(0, c - W) .. c, or 0 .. c when unbounded.  Chunk c' lives in
+// cache slot c' mod S (S = W + 1 for a bounded window, else the chunk
+// capacity), so the visible chunks occupy consecutive slots modulo S and, in
+// slot order, form at most two contiguous token ranges of a head's cache: only
+// the newest chunk may be partly filled (a ragged final chunk), and the ring
+// wrap can split the set once.  Attention does not depend on the order of
+// the keys, so slot order is as good as chunk order.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+#include <new>
+#include <vector>
+
+#include "../../include/fastvr_attn.h"
+#include "fastvr_internal.h"
+
+namespace {
+
+constexpr size_t kControlBytes = 256;
+
+struct Segment {
+  int64_t start, len;
+};
+
+}  // namespace
+
+struct fastvr_plan_s {
+  fastvr_attn_config_t cfg;
+  int64_t slots;         // S
+  int64_t slot_tokens;   // k * N
+  int64_t cache_tokens;  // S * k * N per head
+  size_t kv_bytes;       // bytes of the K region (= the V region)
+  char* base;            // caller's cache buffer
+  int64_t chunks;        // chunks appended since the last reset
+  int32_t last_frames;   // frames of the newest chunk
+  bool device_ready;
+  int device;
+};
+
+namespace {
+
+bool valid_config(const fastvr_attn_config_t* c) {
+  return c != nullptr && c->batch > 0 && c->heads > 0 && c->head_dim > 0 &&
+         c->tokens_per_frame > 0 && c->frames_per_chunk > 0 &&
+         c->window_chunks >= -1 && !(c->softmax_scale < 0.f) &&
+         isfinite(c->softmax_scale) &&
+         (c->window_chunks >= 0 || c->max_chunks > 0);
+}
+
+bool supported_dim(int d) { return d == 64 || d == 128; }
+
+int64_t num_slots(const fastvr_attn_config_t& c) {
+  return c.window_chunks >= 0 ? (int64_t)c.window_chunks + 1 : c.max_chunks;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// Visible segments of the newest chunk, in slot order, merged when adjacent.
+std::vector<Segment> visible_segments(const fastvr_plan_s& p) {
+  std::vector<Segment> segs;
+  const int64_t c = p.chunks - 1;
+  const int32_t W = p.cfg.window_chunks;
+  const int64_t lo = W < 0 ? 0 : std::max<int64_t>(0, c - W);
+  std::vector<Segment> parts;
+  for (int64_t cc = lo; cc <= c; ++cc) {
+    const int64_t slot = cc % p.slots;
+    const int64_t frames = cc == c ? p.last_frames : p.cfg.frames_per_chunk;
+    parts.push_back({slot * p.slot_tokens, frames * p.cfg.tokens_per_frame});
+  }
+  std::sort(parts.begin(), parts.end(),
+            [](const Segment& a, const Segment& b) { return a.start < b.start; });
+  for (const Segment& s : parts) {
+    if (!segs.empty() && segs.back().start + segs.back().len == s.start)
+      segs.back().len += s.len;
+    else
+      segs.push_back(s);
+  }
+  return segs;
+}
+
+fastvr_status_t ensure_device(fastvr_plan_s* p) {
+  if (p->device_ready) return FASTVR_OK;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return FASTVR_ERR_CUDA;
+  int major = 0, minor = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) !=
+          cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  if (major != 10 || minor != 3) return FASTVR_ERR_UNSUPPORTED;
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, p->base) != cudaSuccess ||
+      attr.type != cudaMemoryTypeDevice || attr.device != dev) {
+    cudaGetLastError();
+    return FASTVR_ERR_INVALID_ARG;
+  }
+  // Clear the control block once; kernels only ever set it.
+  if (cudaMemset(p->base + 2 * p->kv_bytes, 0, kControlBytes) != cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  p->device = dev;
+  p->device_ready = true;
+  return FASTVR_OK;
+}
+
+int* control_word(const fastvr_plan_s* p) {
+  return reinterpret_cast<int*>(p->base + 2 * p->kv_bytes);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* fastvr_status_string(fastvr_status_t s) {
+  switch (s) {
+    case FASTVR_OK: return "FASTVR_OK";
+    case FASTVR_ERR_INVALID_ARG: return "FASTVR_ERR_INVALID_ARG";
+    case FASTVR_ERR_UNSUPPORTED: return "FASTVR_ERR_UNSUPPORTED";
+    case FASTVR_ERR_CAPACITY: return "FASTVR_ERR_CAPACITY";
+    case FASTVR_ERR_SEQUENCE: return "FASTVR_ERR_SEQUENCE";
+    case FASTVR_ERR_CUDA: return "FASTVR_ERR_CUDA";
+    case FASTVR_ERR_TIMEOUT: return "FASTVR_ERR_TIMEOUT";
+  }
+  return "FASTVR_ERR_UNKNOWN";
+}
+
+fastvr_status_t fastvr_kv_cache_bytes(const fastvr_attn_config_t* cfg,
+                                      size_t* bytes) {
+  if (!valid_config(cfg) || bytes == nullptr) return FASTVR_ERR_INVALID_ARG;
+  if (!supported_dim(cfg->head_dim)) return FASTVR_ERR_UNSUPPORTED;
+  const int64_t tokens =
+      num_slots(*cfg) * cfg->frames_per_chunk * (int64_t)cfg->tokens_per_frame;
+  const int64_t per = (int64_t)cfg->batch * cfg->heads * tokens * cfg->head_dim * 2;
+  // K and V regions, each a multiple of 256 bytes (d*2 >= 128 and tokens of
+  // a slot are whole rows, so per is a multiple of 128; round up anyway).
+  const int64_t region = (per + 255) / 256 * 256;
+  *bytes = (size_t)(2 * region) + kControlBytes;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_attn_plan(const fastvr_attn_config_t* cfg,
+                                 void* kv_cache, size_t bytes,
+                                 fastvr_plan_t* out) {
+  if (out == nullptr) return FASTVR_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!valid_config(cfg) || kv_cache == nullptr ||
+      ((uintptr_t)kv_cache & 255u) != 0)
+    return FASTVR_ERR_INVALID_ARG;
+  if (!supported_dim(cfg->head_dim)) return FASTVR_ERR_UNSUPPORTED;
+  size_t need = 0;
+  fastvr_status_t st = fastvr_kv_cache_bytes(cfg, &need);
+  if (st != FASTVR_OK) return st;
+  if (bytes < need) return FASTVR_ERR_CAPACITY;
+  fastvr_plan_s* p = new (std::nothrow) fastvr_plan_s();
+  if (p == nullptr) return FASTVR_ERR_INVALID_ARG;
+  p->cfg = *cfg;
+  if (p->cfg.softmax_scale == 0.f)
+    p->cfg.softmax_scale = 1.f / sqrtf((float)cfg->head_dim);
+  if (p->cfg.window_chunks >= 0) p->cfg.max_chunks = 0;
+  p->slots = num_slots(*cfg);
+  p->slot_tokens = (int64_t)cfg->frames_per_chunk * cfg->tokens_per_frame;
+  p->cache_tokens = p->slots * p->slot_tokens;
+  p->kv_bytes = (need - kControlBytes) / 2;
+  p->base = static_cast<char*>(kv_cache);
+  p->chunks = 0;
+  p->last_frames = 0;
+  p->device_ready = false;
+  p->device = -1;
+  *out = p;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_kv_append(fastvr_plan_t p, const void* k_new,
+                                 const void* v_new, int32_t frames,
+                                 struct CUstream_st* stream) {
+  if (p == nullptr || k_new == nullptr || v_new == nullptr || frames < 1 ||
+      !aligned16(k_new) || !aligned16(v_new))
+    return FASTVR_ERR_INVALID_ARG;
+  if (frames > p->cfg.frames_per_chunk) return FASTVR_ERR_CAPACITY;
+  if (p->chunks > 0 && p->last_frames < p->cfg.frames_per_chunk)
+    return FASTVR_ERR_SEQUENCE;  // the stream already ended with a ragged chunk
+  if (p->cfg.window_chunks < 0 && p->chunks >= p->cfg.max_chunks)
+    return FASTVR_ERR_CAPACITY;
+  fastvr_status_t st = ensure_device(p);
+  if (st != FASTVR_OK) return st;
+
+  fastvr::AppendParams a;
+  a.k_new = static_cast<const uint16_t*>(k_new);
+  a.v_new = static_cast<const uint16_t*>(v_new);
+  a.k_cache = reinterpret_cast<uint16_t*>(p->base);
+  a.v_cache = reinterpret_cast<uint16_t*>(p->base + p->kv_bytes);
+  a.batch = p->cfg.batch;
+  a.tokens = frames * p->cfg.tokens_per_frame;
+  a.heads = p->cfg.heads;
+  a.head_dim = p->cfg.head_dim;
+  a.cache_tokens = p->cache_tokens;
+  a.token_offset = (p->chunks % p->slots) * p->slot_tokens;
+  if (fastvr::launch_kv_append(a, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  p->chunks += 1;
+  p->last_frames = frames;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_chunk_attn_fwd(fastvr_plan_t p, const void* q, void* out,
+                                      float* lse, struct CUstream_st* stream) {
+  if (p == nullptr || q == nullptr || out == nullptr || !aligned16(q) ||
+      !aligned16(out) || (((uintptr_t)lse) & 3u) != 0)
+    return FASTVR_ERR_INVALID_ARG;
+  if (p->chunks == 0) return FASTVR_ERR_SEQUENCE;
+  fastvr_status_t st = ensure_device(p);
+  if (st != FASTVR_OK) return st;
+
+  const std::vector<Segment> segs = visible_segments(*p);
+  if ((int)segs.size() > fastvr::kMaxSegments) return FASTVR_ERR_INVALID_ARG;
+  const fastvr_attn_config_t& c = p->cfg;
+  fastvr::AttnParams a;
+  memset(&a, 0, sizeof(a));
+  a.q = static_cast<const uint16_t*>(q);
+  a.o = static_cast<uint16_t*>(out);
+  a.lse = lse;
+  a.k = reinterpret_cast<const uint16_t*>(p->base);
+  a.v = reinterpret_cast<const uint16_t*>(p->base + p->kv_bytes);
+  a.batch = c.batch;
+  a.heads = c.heads;
+  a.head_dim = c.head_dim;
+  a.q_tokens = p->last_frames * c.tokens_per_frame;
+  a.q_str.head = c.head_dim;
+  a.q_str.token = (int64_t)c.heads * c.head_dim;
+  a.q_str.batch = (int64_t)a.q_tokens * c.heads * c.head_dim;
+  a.kv_str.token = c.head_dim;
+  a.kv_str.head = p->cache_tokens * c.head_dim;
+  a.kv_str.batch = (int64_t)c.heads * p->cache_tokens * c.head_dim;
+  a.kv_tokens = p->cache_tokens;
+  a.num_segments = (int32_t)segs.size();
+  for (size_t i = 0; i < segs.size(); ++i) {
+    a.seg_start[i] = segs[i].start;
+    a.seg_len[i] = (int32_t)segs[i].len;
+  }
+  a.scale_log2 = c.softmax_scale * 1.4426950408889634f;
+  a.status = control_word(p);
+  if (fastvr::launch_chunk_attn(a, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_plan_reset(fastvr_plan_t p) {
+  if (p == nullptr) return FASTVR_ERR_INVALID_ARG;
+  p->chunks = 0;
+  p->last_frames = 0;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_get_status(fastvr_plan_t p) {
+  if (p == nullptr) return FASTVR_ERR_INVALID_ARG;
+  if (!p->device_ready) return FASTVR_OK;
+  if (cudaDeviceSynchronize() != cudaSuccess) return FASTVR_ERR_CUDA;
+  int word = 0;
+  if (cudaMemcpy(&word, control_word(p), sizeof(int), cudaMemcpyDeviceToHost) !=
+      cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  if (word != fastvr::kDevOk) {
+    const int zero = 0;
+    cudaMemcpy(control_word(p), &zero, sizeof(int), cudaMemcpyHostToDevice);
+    return FASTVR_ERR_TIMEOUT;
+  }
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_plan_get_state(fastvr_plan_t p, int64_t* chunks,
+                                      int32_t* last_frames) {
+  if (p == nullptr || chunks == nullptr || last_frames == nullptr)
+    return FASTVR_ERR_INVALID_ARG;
+  *chunks = p->chunks;
+  *last_frames = p->last_frames;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_plan_set_state(fastvr_plan_t p, int64_t chunks,
+                                      int32_t last_frames) {
+  if (p == nullptr || chunks < 0) return FASTVR_ERR_INVALID_ARG;
+  if (chunks == 0 ? last_frames != 0
+                  : (last_frames < 1 || last_frames > p->cfg.frames_per_chunk))
+    return FASTVR_ERR_INVALID_ARG;
+  if (p->cfg.window_chunks < 0 && chunks > p->cfg.max_chunks)
+    return FASTVR_ERR_CAPACITY;
+  p->chunks = chunks;
+  p->last_frames = last_frames;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_plan_visible(fastvr_plan_t p, int32_t* num_segments,
+                                    int64_t* seg_start, int64_t* seg_len,
+                                    int64_t* visible_tokens) {
+  if (p == nullptr || num_segments == nullptr || seg_start == nullptr ||
+      seg_len == nullptr || visible_tokens == nullptr)
+    return FASTVR_ERR_INVALID_ARG;
+  if (p->chunks == 0) return FASTVR_ERR_SEQUENCE;
+  const std::vector<Segment> segs = visible_segments(*p);
+  if ((int)segs.size() > fastvr::kMaxSegments) return FASTVR_ERR_INVALID_ARG;
+  int64_t total = 0;
+  for (size_t i = 0; i < segs.size(); ++i) {
+    seg_start[i] = segs[i].start;
+    seg_len[i] = segs[i].len;
+    total += segs[i].len;
+  }
+  *num_segments = (int32_t)segs.size();
+  *visible_tokens = total;
+  return FASTVR_OK;
+}
+
+void fastvr_plan_destroy(fastvr_plan_t p) { delete p; }
+
+}  // extern "C"

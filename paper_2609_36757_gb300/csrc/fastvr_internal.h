@@ -1,0 +1,57 @@
+// Internal interfaces between the host library (fastvr_host.cpp) and the
+// CUDA kernels.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace fastvr {
+
+// At most two contiguous token ranges of one head's cache make up the keys a
+// chunk sees: the visible chunk slots are consecutive modulo the ring size
+// and only the newest chunk can be partly filled (Eq. 1 at chunk granularity,
+// Sec. 3.1 KV caching).
+constexpr int kMaxSegments = 2;
+
+// Error codes a kernel writes into the cache's control block.
+constexpr int kDevOk = 0;
+constexpr int kDevTimeout = 1;
+
+// Strided view of a bfloat16 [B, L, H, d] token-major tensor or of a head-major
+// cache [B, H, L, d]: element (b, t, h, x) lives at
+// base + b*batch + t*token + h*head + x (strides in elements).
+struct Strides {
+  int64_t batch, token, head;
+};
+
+struct AppendParams {
+  const uint16_t* k_new;  // [B, L, H, d] token-major
+  const uint16_t* v_new;
+  uint16_t* k_cache;      // [B, H, cache_tokens, d] head-major
+  uint16_t* v_cache;
+  int32_t batch, tokens, heads, head_dim;
+  int64_t cache_tokens;   // tokens per head in the cache (S * k * N)
+  int64_t token_offset;   // first cache token of the destination slot
+};
+
+struct AttnParams {
+  const uint16_t* q;      // bfloat16 [B, Lq, H, d] token-major
+  uint16_t* o;            // bfloat16 [B, Lq, H, d] token-major
+  float* lse;             // float32 [B, H, Lq] or null
+  const uint16_t* k;      // keys: head-major cache view
+  const uint16_t* v;      // values: same layout as k
+  Strides q_str;          // strides of q and o
+  Strides kv_str;         // strides of k and v
+  int32_t batch, heads, head_dim, q_tokens;
+  int64_t kv_tokens;      // tokens per head addressable through k/v
+  int32_t num_segments;
+  int64_t seg_start[kMaxSegments];
+  int32_t seg_len[kMaxSegments];
+  float scale_log2;       // softmax_scale * log2(e)
+  int* status;            // control word (device)
+};
+
+cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream);
+cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream);
+
+}  // namespace fastvr

@@ -1,0 +1,152 @@
+"""GPU parity: the library's kernels (through the C ABI) against the CPU
+oracle on the same seeded bf16 inputs."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import attention as OA
+from oracle import kv_cache as OK
+from paper_2609_36757_gb300 import workloads as WL
+from parity_helpers import Err, run_stream, to64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def FV():
+    from paper_2609_36757_gb300 import fastvr
+    return fastvr
+
+
+# ------------------------------------------------------------- KV append
+@pytest.mark.parametrize("w", [
+    WL.custom("ring", batch=2, heads=3, head_dim=64, tokens_per_frame=5,
+              frames_per_chunk=2, num_chunks=6, window_chunks=1,
+              last_chunk_frames=1, seed=11),
+    WL.custom("unbounded", batch=1, heads=12, head_dim=128,
+              tokens_per_frame=1590, frames_per_chunk=2, num_chunks=4,
+              seed=12),
+    WL.custom("w0", batch=1, heads=2, head_dim=128, tokens_per_frame=77,
+              frames_per_chunk=3, num_chunks=4, window_chunks=0,
+              last_chunk_frames=2, seed=13),
+], ids=lambda w: w.name)
+def test_kv_append_is_bit_exact(FV, w):
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    att.cache.fill_(0x5A)
+    ref = OK.RingCache(w.batch, w.heads, w.head_dim, w.tokens_per_frame,
+                       w.frames_per_chunk, w.window_chunks, w.max_chunks,
+                       fill=0x5A5A)
+    region = ref.k.size * 2
+    for c, q, k, v in WL.chunk_stream(w):
+        att.append(k.cuda(), v.cuda())
+        ref.append(k.view(torch.int16).numpy().view(np.uint16),
+                   v.view(torch.int16).numpy().view(np.uint16))
+        torch.cuda.synchronize()
+        raw = att.cache.cpu().numpy()
+        got_k = raw[:region].view(np.uint16).reshape(ref.k.shape)
+        got_v = raw[region:2 * region].view(np.uint16).reshape(ref.v.shape)
+        assert np.array_equal(got_k, ref.k), f"K differs after chunk {c}"
+        assert np.array_equal(got_v, ref.v), f"V differs after chunk {c}"
+
+
+# ------------------------------------------------- small streams, every element
+SMALL = [
+    # several 128-row Q tiles with a ragged tail, several key tiles per segment
+    WL.custom("N300-k2", batch=1, heads=2, head_dim=128, tokens_per_frame=300,
+              frames_per_chunk=2, num_chunks=4, seed=21),
+    WL.custom("N97-k3-W1", batch=2, heads=3, head_dim=128, tokens_per_frame=97,
+              frames_per_chunk=3, num_chunks=6, window_chunks=1,
+              last_chunk_frames=2, seed=22),
+    WL.custom("d64-N130-W2", batch=1, heads=4, head_dim=64,
+              tokens_per_frame=130, frames_per_chunk=2, num_chunks=5,
+              window_chunks=2, last_chunk_frames=1, seed=23),
+    WL.custom("W0", batch=1, heads=2, head_dim=128, tokens_per_frame=200,
+              frames_per_chunk=1, num_chunks=4, window_chunks=0, seed=24),
+    WL.custom("N1-k1", batch=1, heads=2, head_dim=64, tokens_per_frame=1,
+              frames_per_chunk=1, num_chunks=9, seed=25),
+    WL.custom("peaked", batch=1, heads=2, head_dim=128, tokens_per_frame=250,
+              frames_per_chunk=2, num_chunks=3, seed=26, peaked=True),
+    WL.custom("ring-wrap", batch=1, heads=2, head_dim=128, tokens_per_frame=64,
+              frames_per_chunk=2, num_chunks=9, window_chunks=3,
+              last_chunk_frames=1, seed=27),
+]
+
+
+@pytest.mark.parametrize("w", SMALL, ids=lambda w: w.name)
+def test_small_stream_every_element(w):
+    err = run_stream(w)
+    err.check()
+
+
+@pytest.mark.parametrize("w", SMALL[:3], ids=lambda w: w.name)
+def test_streamed_gpu_equals_oneshot_oracle(FV, w):
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    qs, ks, vs, outs, lses = [], [], [], [], []
+    for c, q, k, v in WL.chunk_stream(w):
+        att.append(k.cuda(), v.cuda())
+        o, l = att.forward(q.cuda(), want_lse=True)
+        qs.append(q), ks.append(k), vs.append(v)
+        outs.append(o.cpu()), lses.append(l.cpu())
+    ref_o, ref_l = OA.blockcausal_attention(
+        to64(torch.cat(qs, 1)), to64(torch.cat(ks, 1)), to64(torch.cat(vs, 1)),
+        w.tokens_per_frame, w.frames_per_chunk, w.window_chunks,
+        w.softmax_scale)
+    err = Err()
+    err.add(to64(torch.cat(outs, 1)), ref_o, torch.cat(lses, 2).numpy(), ref_l)
+    err.check()
+
+
+def test_forward_is_deterministic_and_repeatable(FV):
+    w = SMALL[1]
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    for c, q, k, v in WL.chunk_stream(w):
+        att.append(k.cuda(), v.cuda())
+        qd = q.cuda()
+        o1 = att.forward(qd)
+        o2 = att.forward(qd)
+        assert torch.equal(o1, o2)
+
+
+def test_errors_on_the_gpu_path(FV):
+    w = SMALL[1]
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    q = torch.zeros(w.chunk_shape(0), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(FV.FastVRError) as e:
+        att.forward(q)
+    assert e.value.status == FV.FASTVR_ERR_SEQUENCE
+    att.append(q, q)
+    ragged = q[:, :w.tokens_per_frame].contiguous()
+    att.append(ragged, ragged)
+    with pytest.raises(FV.FastVRError) as e:
+        att.append(q, q)
+    assert e.value.status == FV.FASTVR_ERR_SEQUENCE
+    assert att.status() == FV.FASTVR_OK
+
+
+# ------------------------------------------------------- the five workloads
+def test_workload_tiny_every_element():
+    run_stream(WL.TINY).check()
+
+
+def test_workload_480p_every_element():
+    run_stream(WL.W480P).check()
+
+
+def test_workload_720p_peaked_sampled_rows():
+    run_stream(WL.W720P_PEAKED, rows_per_chunk=256).check()
+
+
+def test_workload_1080p_sampled_rows():
+    run_stream(WL.W1080P, rows_per_chunk=48).check()
+
+
+def test_workload_1080p_windowed_sampled_rows():
+    run_stream(WL.W1080P_WINDOWED, rows_per_chunk=12, chunk_stride=4).check()
+
+
+def test_paper_window_eq1_k3_w1_sampled_rows():
+    # Eq. 1 as printed: each chunk sees itself and one predecessor, k = 3
+    w = WL.custom("eq1-k3-W1", batch=1, heads=4, head_dim=128,
+                  tokens_per_frame=8160, frames_per_chunk=3, num_chunks=5,
+                  window_chunks=1, last_chunk_frames=2, seed=31)
+    run_stream(w, rows_per_chunk=32).check()
