@@ -1,22 +1,97 @@
-// Chunk-causal attention forward (Sec. 3.1, Eq. 1), first GPU kernel.
+// Chunk-causal attention forward for sm_103a (Sec. 3.1, Eq. 1): tcgen05
+// tensor cores with TMEM accumulators, TMA-staged tiles, fp32 online softmax.
 //
-// One CTA computes 128 query rows of one (batch, head) against the visible
-// key segments of the cache, with an online softmax in float32 (exp2 domain)
-// and bf16 tensor-core MMAs (m16n8k16) accumulating in float32.  Masking
-// happens at chunk granularity, so every key inside a visible segment is
-// visible to every query of the chunk; the only in-kernel mask is the ragged
-// end of a segment, whose tail columns are set to -inf.
+// Masking acts at chunk granularity and a call attends one chunk's queries,
+// so every key of the visible segments is visible to every query: the host
+// enumerates only visible cache ranges (block-causal skipping happens before
+// launch, invisible chunks are never loaded) and the only in-kernel mask is
+// the ragged end of a segment.
+//
+// One CTA owns two 128-row query tiles of one (batch, head) and streams the
+// visible keys in 128-key tiles:
+//   warp 8      TMA producer: Q tiles once, then K and V tiles through
+//               two-stage rings (128-byte swizzled boxes of 64 columns).
+//   warp 9      MMA issuer (one thread): S_t = Q_t K^T into TMEM, then
+//               O_t += P_t V with P_t read from TMEM.
+//   warps 0-3   softmax of query tile 0, one thread per row (TMEM lane);
+//   warps 4-7   softmax of query tile 1.
+// TMEM (512 columns): S_0 | S_1 | O_0 | O_1, 128 columns each; P_t (bf16
+// pairs, 64 columns) overwrites the first half of S_t once S_t is in
+// registers.  The two query tiles alternate on the tensor pipe, so one
+// tile's softmax overlaps the other tile's MMAs.
+//
+// Online softmax in the exp2 domain: each row keeps a reference m (a lower
+// bound of its running max) and exponentiates against it; m moves, and O is
+// rescaled, only when a tile's max exceeds m by more than 8 (P stays <= 256,
+// finite in bf16 and fp32).  The final O / l is the same for any reference,
+// so this is exact up to rounding.  When S_t(j) is ready, PV_t(j-1) has
+// completed too (one commit tracks every earlier MMA), so the rescale needs
+// no extra wait.
+//
+// Every mbarrier wait is bounded: past the limit the kernel records
+// FASTVR timeout in the control word, all roles stop issuing, in-flight TMA
+// loads and MMAs are drained, TMEM is released and the CTA exits.
+#include <cuda.h>
 #include <cuda_bf16.h>
+#include <math.h>
 
 #include "fastvr_internal.h"
+#include "sm100_ptx.cuh"
 
 namespace fastvr {
 namespace {
 
-constexpr int kBlockM = 128;  // query rows per CTA (16 per warp)
-constexpr int kBlockN = 64;   // keys per tile
-constexpr int kWarps = 8;
-constexpr int kThreads = kWarps * 32;
+using namespace sm100;
+
+constexpr int kBM = 128;        // query rows per tile (one TMEM lane each)
+constexpr int kBN = 128;        // keys per tile
+constexpr int kQTiles = 2;      // query tiles per CTA
+constexpr int kStages = 2;      // depth of the K and V rings
+constexpr int kThreads = 320;   // 8 softmax warps + producer + MMA warp
+constexpr int kBox = 128 * 128; // one TMA box: 128 rows x 64 bf16 (bytes)
+constexpr uint32_t kTmemCols = 512;
+constexpr float kRescaleThreshold = 8.0f;      // log2 units
+constexpr uint64_t kWaitLimitNs = 4000000000ull;  // 4 s per wait
+
+struct TcParams {
+  CUtensorMap q_map;                  // {d, Lq, H, B}
+  CUtensorMap k_map[kMaxSegments];    // {d, segment end, H, B} of the cache
+  CUtensorMap v_map[kMaxSegments];
+  uint16_t* o;
+  float* lse;
+  Strides o_str;
+  int32_t q_tokens, heads;
+  int32_t seg_start[kMaxSegments];
+  int32_t seg_len[kMaxSegments];
+  int32_t seg_tiles0;   // tiles of segment 0
+  int32_t total_tiles;
+  float scale_log2;
+  int* status;
+};
+
+struct Shared {
+  uint64_t q_full;
+  uint64_t k_full[kStages], k_empty[kStages];
+  uint64_t v_full[kStages], v_empty[kStages];
+  uint64_t s_full[kQTiles], p_full[kQTiles];
+  uint64_t o_full, drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+template <int D>
+struct Layout {
+  static constexpr int kNB = D / 64;  // boxes per tile
+  __host__ __device__ static constexpr int q(int t, int bx) { return (t * kNB + bx) * kBox; }
+  __host__ __device__ static constexpr int k(int s, int bx) {
+    return ((kQTiles + s) * kNB + bx) * kBox;
+  }
+  __host__ __device__ static constexpr int v(int s, int bx) {
+    return ((kQTiles + kStages + s) * kNB + bx) * kBox;
+  }
+  static constexpr int shared_off = (kQTiles + 2 * kStages) * kNB * kBox;
+  static constexpr int bytes = shared_off + 1024 /*Shared*/ + 1024 /*align*/;
+};
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -24,277 +99,400 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src,
-                                           bool valid) {
-  const int n = valid ? 16 : 0;  // zero-fill when the row is out of range
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst),
-               "l"(src), "r"(n));
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;\n" ::);
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0,
-                                        uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0,
-                                          uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile(
-      "ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-      : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-      : "r"(addr));
-}
-
-__device__ __forceinline__ void mma_bf16(float* c, const uint32_t* a,
-                                         uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Locate tile `it` of the flattened visible segment list.
-__device__ __forceinline__ void tile_at(const AttnParams& p, int it,
-                                        int64_t& tok0, int& valid) {
-  for (int s = 0; s < p.num_segments; ++s) {
-    const int tiles = (p.seg_len[s] + kBlockN - 1) / kBlockN;
-    if (it < tiles) {
-      tok0 = p.seg_start[s] + (int64_t)it * kBlockN;
-      valid = min(kBlockN, p.seg_len[s] - it * kBlockN);
-      return;
+// Bounded wait.  Returns false when this wait timed out or another role
+// already aborted; the first timeout records the error.
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
+                                      Shared* S, int* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*reinterpret_cast<volatile int*>(&S->abort)) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      *reinterpret_cast<volatile int*>(&S->abort) = 1;
+      atomicExch(status, kDevTimeout);
+      return false;
     }
-    it -= tiles;
   }
-  tok0 = 0;
-  valid = 0;
+}
+
+// Bounded wait that ignores the abort flag (draining in-flight work).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > kWaitLimitNs) return;
+  }
+}
+
+__device__ __forceinline__ void tile_coord(const TcParams& p, int j, int& seg,
+                                           int& tok0, int& valid) {
+  seg = j < p.seg_tiles0 ? 0 : 1;
+  const int jj = seg ? j - p.seg_tiles0 : j;
+  tok0 = p.seg_start[seg] + jj * kBN;
+  valid = min(kBN, p.seg_len[seg] - jj * kBN);
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads)
-chunk_attn_mma_kernel(const AttnParams p) {
-  constexpr int kStride = D + 8;  // padded smem row (elements): no conflicts
-  constexpr int kChunks = D / 8;  // 16-byte pieces per row
-  extern __shared__ __align__(16) uint16_t smem[];
-  uint16_t* sQ = smem;                          // [kBlockM][kStride]
-  uint16_t* sK = sQ + kBlockM * kStride;        // [2][kBlockN][kStride]
-  uint16_t* sV = sK + 2 * kBlockN * kStride;    // [2][kBlockN][kStride]
-
-  const int tid = threadIdx.x, warp = tid / 32, lane = tid % 32;
-  const int q0 = blockIdx.x * kBlockM;
-  const int h = blockIdx.y, b = blockIdx.z;
-
-  const uint16_t* qbase = p.q + b * p.q_str.batch + h * p.q_str.head;
-  const uint16_t* kbase = p.k + b * p.kv_str.batch + h * p.kv_str.head;
-  const uint16_t* vbase = p.v + b * p.kv_str.batch + h * p.kv_str.head;
-
-  int num_tiles = 0;
-  for (int s = 0; s < p.num_segments; ++s)
-    num_tiles += (p.seg_len[s] + kBlockN - 1) / kBlockN;
-
-  // Q tile (zero rows past the end of the chunk).
-  for (int i = tid; i < kBlockM * kChunks; i += kThreads) {
-    const int r = i / kChunks, c = i % kChunks;
-    const bool ok = q0 + r < p.q_tokens;
-    const uint16_t* src = qbase + (int64_t)(ok ? q0 + r : 0) * p.q_str.token + c * 8;
-    cp_async16(smem_u32(sQ + r * kStride + c * 8), src, ok);
+__device__ void producer(const TcParams& p, uint8_t* smem, Shared* S, int q0,
+                         int h, int b) {
+  using L = Layout<D>;
+  tma_prefetch_desc(&p.q_map);
+  for (int s = 0; s < kMaxSegments; ++s) {
+    tma_prefetch_desc(&p.k_map[s]);
+    tma_prefetch_desc(&p.v_map[s]);
   }
-  cp_async_commit();
+  mbar_arrive_expect_tx(&S->q_full, kQTiles * L::kNB * kBox);
+  for (int t = 0; t < kQTiles; ++t)
+    for (int bx = 0; bx < L::kNB; ++bx)
+      tma_load_4d(&p.q_map, smem + L::q(t, bx), &S->q_full, bx * 64,
+                  q0 + t * kBM, h, b);
+  int nk = 0, nv = 0;
+  for (int j = 0; j < p.total_tiles; ++j) {
+    const int st = j % kStages;
+    const uint32_t ph = (j / kStages) & 1;
+    int seg, tok0, valid;
+    tile_coord(p, j, seg, tok0, valid);
+    if (!wait_bar(&S->k_empty[st], ph ^ 1, S, p.status)) break;
+    mbar_arrive_expect_tx(&S->k_full[st], L::kNB * kBox);
+    for (int bx = 0; bx < L::kNB; ++bx)
+      tma_load_4d(&p.k_map[seg], smem + L::k(st, bx), &S->k_full[st], bx * 64,
+                  tok0, h, b);
+    ++nk;
+    if (!wait_bar(&S->v_empty[st], ph ^ 1, S, p.status)) break;
+    mbar_arrive_expect_tx(&S->v_full[st], L::kNB * kBox);
+    for (int bx = 0; bx < L::kNB; ++bx)
+      tma_load_4d(&p.v_map[seg], smem + L::v(st, bx), &S->v_full[st], bx * 64,
+                  tok0, h, b);
+    ++nv;
+  }
+  // Every issued load has landed before the CTA may exit (a no-op wait in
+  // normal operation: consumers already waited for them).
+  drain_wait(&S->q_full, 0);
+  for (int i = max(0, nk - kStages); i < nk; ++i)
+    drain_wait(&S->k_full[i % kStages], (i / kStages) & 1);
+  for (int i = max(0, nv - kStages); i < nv; ++i)
+    drain_wait(&S->v_full[i % kStages], (i / kStages) & 1);
+}
 
-  auto load_kv = [&](int it, int stage) {
-    int64_t tok0;
-    int valid;
-    tile_at(p, it, tok0, valid);
-    uint16_t* dk = sK + stage * kBlockN * kStride;
-    uint16_t* dv = sV + stage * kBlockN * kStride;
-    for (int i = tid; i < kBlockN * kChunks; i += kThreads) {
-      const int r = i / kChunks, c = i % kChunks;
-      const int64_t t = tok0 + r;
-      const bool ok = r < valid && t < p.kv_tokens;
-      const int64_t off = (ok ? t : 0) * p.kv_str.token + c * 8;
-      cp_async16(smem_u32(dk + r * kStride + c * 8), kbase + off, ok);
-      cp_async16(smem_u32(dv + r * kStride + c * 8), vbase + off, ok);
+template <int D>
+__device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
+                           uint32_t tmem) {
+  using L = Layout<D>;
+  constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, 0);
+  constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, D, 1);
+  const uint32_t sbase = smem_addr(smem);
+  const int n = p.total_tiles;
+
+  // S_t = Q_t K^T: both operands K-major, 128-byte swizzle; a K step of 16
+  // elements is 32 bytes inside a 64-column box.
+  auto qk = [&](int t, int st) {
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+      const uint32_t off = (ks / 4) * kBox + (ks % 4) * 32;
+      const uint64_t a = smem_desc_sw128(sbase + L::q(t, 0) + off, 16, 1024);
+      const uint64_t bdesc = smem_desc_sw128(sbase + L::k(st, 0) + off, 16, 1024);
+      mma_ss(tmem + t * 128, a, bdesc, kIdescQK, ks > 0);
+    }
+  };
+  // O_t += P_t V: P_t from TMEM (8 columns per 16 keys), V MN-major (d
+  // contiguous): 16 keys are two 8-row groups (2048 bytes), the two 64-column
+  // halves of d are one box apart.
+  auto pv = [&](int t, int st, int acc) {
+#pragma unroll
+    for (int kk = 0; kk < kBN / 16; ++kk) {
+      const uint64_t bdesc =
+          smem_desc_sw128(sbase + L::v(st, 0) + kk * 2048, kBox, 1024);
+      mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, bdesc, kIdescPV,
+             (acc | kk) != 0);
     }
   };
 
-  if (num_tiles > 0) load_kv(0, 0);
-  cp_async_commit();
-
-  // Q fragments stay in registers for the whole key stream.
-  cp_async_wait<1>();
-  __syncthreads();
-  uint32_t qf[D / 16][4];
-  {
-    const int row = warp * 16 + (lane % 16);
-    const int col = (lane / 16) * 8;
-#pragma unroll
-    for (int ks = 0; ks < D / 16; ++ks)
-      ldsm_x4(smem_u32(sQ + row * kStride + ks * 16 + col), qf[ks][0],
-              qf[ks][1], qf[ks][2], qf[ks][3]);
+  bool ok = wait_bar(&S->q_full, 0, S, p.status) &&
+            wait_bar(&S->k_full[0], 0, S, p.status);
+  if (ok) {
+    tc_fence_after();
+    qk(0, 0);
+    mma_commit(&S->s_full[0]);
+    qk(1, 0);
+    mma_commit(&S->s_full[1]);
+    mma_commit(&S->k_empty[0]);
   }
-
-  float o_acc[D / 8][4];
-#pragma unroll
-  for (int j = 0; j < D / 8; ++j)
-    o_acc[j][0] = o_acc[j][1] = o_acc[j][2] = o_acc[j][3] = 0.f;
-  float m_run[2] = {-INFINITY, -INFINITY};  // exp2-domain running max
-  float l_run[2] = {0.f, 0.f};              // per-thread partial sums
-
-  const int g = lane / 4, t4 = lane % 4;
-  for (int it = 0; it < num_tiles; ++it) {
-    if (it + 1 < num_tiles) load_kv(it + 1, (it + 1) & 1);
-    cp_async_commit();
-    cp_async_wait<1>();
-    __syncthreads();
-
-    int64_t tok0;
-    int valid;
-    tile_at(p, it, tok0, valid);
-    const uint16_t* k_s = sK + (it & 1) * kBlockN * kStride;
-    const uint16_t* v_s = sV + (it & 1) * kBlockN * kStride;
-
-    // S = Q K^T for this warp's 16 rows x 64 keys.
-    float s[kBlockN / 8][4];
-#pragma unroll
-    for (int n = 0; n < kBlockN / 8; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
-#pragma unroll
-    for (int ks = 0; ks < D / 16; ++ks) {
-#pragma unroll
-      for (int n2 = 0; n2 < kBlockN / 16; ++n2) {
-        const int mi = lane / 8, rr = lane % 8;
-        const int row = n2 * 16 + (mi / 2) * 8 + rr;
-        const int col = ks * 16 + (mi % 2) * 8;
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(smem_u32(k_s + row * kStride + col), b0, b1, b2, b3);
-        mma_bf16(s[2 * n2], qf[ks], b0, b1);
-        mma_bf16(s[2 * n2 + 1], qf[ks], b2, b3);
-      }
+  for (int j = 0; ok && j < n; ++j) {
+    const int st = j % kStages;
+    const uint32_t ph = (j / kStages) & 1;
+    const int jn = j + 1;
+    const int stn = jn % kStages;
+    const uint32_t phn = (jn / kStages) & 1;
+    if (!(ok = wait_bar(&S->v_full[st], ph, S, p.status))) break;
+    if (!(ok = wait_bar(&S->p_full[0], j & 1, S, p.status))) break;
+    tc_fence_after();
+    pv(0, st, j > 0);
+    if (jn < n) {
+      if (!(ok = wait_bar(&S->k_full[stn], phn, S, p.status))) break;
+      tc_fence_after();
+      qk(0, stn);
+      mma_commit(&S->s_full[0]);
     }
-
-    // Online softmax over the tile (rows g and g + 8 of this warp).
-    float mx[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-    for (int n = 0; n < kBlockN / 8; ++n) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int col = n * 8 + 2 * t4 + (e & 1);
-        float x = s[n][e] * p.scale_log2;
-        if (col >= valid) x = -INFINITY;
-        s[n][e] = x;
-        mx[e >> 1] = fmaxf(mx[e >> 1], x);
-      }
+    if (!(ok = wait_bar(&S->p_full[1], j & 1, S, p.status))) break;
+    tc_fence_after();
+    pv(1, st, j > 0);
+    mma_commit(&S->v_empty[st]);
+    if (jn < n) {
+      qk(1, stn);
+      mma_commit(&S->s_full[1]);
+      mma_commit(&S->k_empty[stn]);
     }
-    float alpha[2];
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
-      const float m_new = fmaxf(m_run[r], mx[r]);
-      alpha[r] = ex2(m_run[r] - m_new);
-      m_run[r] = m_new;
-      l_run[r] *= alpha[r];
-    }
-#pragma unroll
-    for (int n = 0; n < kBlockN / 8; ++n) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float pe = ex2(s[n][e] - m_run[e >> 1]);
-        s[n][e] = pe;
-        l_run[e >> 1] += pe;
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < D / 8; ++j) {
-      o_acc[j][0] *= alpha[0];
-      o_acc[j][1] *= alpha[0];
-      o_acc[j][2] *= alpha[1];
-      o_acc[j][3] *= alpha[1];
-    }
-
-    // O += P V.
-#pragma unroll
-    for (int kk = 0; kk < kBlockN / 16; ++kk) {
-      uint32_t a[4];
-      a[0] = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
-      a[1] = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
-      a[2] = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-      a[3] = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-      for (int n2 = 0; n2 < D / 16; ++n2) {
-        const int mi = lane / 8, rr = lane % 8;
-        const int row = kk * 16 + (mi % 2) * 8 + rr;
-        const int col = n2 * 16 + (mi / 2) * 8;
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(smem_u32(v_s + row * kStride + col), b0, b1, b2, b3);
-        mma_bf16(o_acc[2 * n2], a, b0, b1);
-        mma_bf16(o_acc[2 * n2 + 1], a, b2, b3);
-      }
-    }
-    __syncthreads();  // stage (it & 1) is refilled by the next iteration
   }
-
-  // Epilogue: normalise, stage through shared memory, store coalesced.
-  float inv_l[2];
-#pragma unroll
-  for (int r = 0; r < 2; ++r) {
-    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 1);
-    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 2);
-    inv_l[r] = 1.f / l_run[r];
-  }
-  const int r0 = warp * 16 + g;
-#pragma unroll
-  for (int j = 0; j < D / 8; ++j) {
-    const int col = j * 8 + 2 * t4;
-    *reinterpret_cast<uint32_t*>(sQ + r0 * kStride + col) =
-        pack_bf16(o_acc[j][0] * inv_l[0], o_acc[j][1] * inv_l[0]);
-    *reinterpret_cast<uint32_t*>(sQ + (r0 + 8) * kStride + col) =
-        pack_bf16(o_acc[j][2] * inv_l[1], o_acc[j][3] * inv_l[1]);
-  }
-  if (p.lse != nullptr && t4 == 0) {
-    float* lse = p.lse + ((int64_t)b * p.heads + h) * p.q_tokens;
-    const float ln2 = 0.6931471805599453f;
-    if (q0 + r0 < p.q_tokens) lse[q0 + r0] = (m_run[0] + __log2f(l_run[0])) * ln2;
-    if (q0 + r0 + 8 < p.q_tokens)
-      lse[q0 + r0 + 8] = (m_run[1] + __log2f(l_run[1])) * ln2;
-  }
-  __syncthreads();
-  uint16_t* obase = p.o + b * p.q_str.batch + h * p.q_str.head;
-  for (int i = tid; i < kBlockM * kChunks; i += kThreads) {
-    const int r = i / kChunks, c = i % kChunks;
-    if (q0 + r < p.q_tokens)
-      *reinterpret_cast<uint4*>(obase + (int64_t)(q0 + r) * p.q_str.token + c * 8) =
-          *reinterpret_cast<const uint4*>(sQ + r * kStride + c * 8);
-  }
+  if (ok) mma_commit(&S->o_full);
+  mma_commit(&S->drain);
+  drain_wait(&S->drain, 0);
 }
 
 template <int D>
-cudaError_t launch_d(const AttnParams& p, cudaStream_t stream) {
-  constexpr int kStride = D + 8;
-  const size_t smem = (size_t)(kBlockM + 4 * kBlockN) * kStride * sizeof(uint16_t);
-  cudaError_t e = cudaFuncSetAttribute(chunk_attn_mma_kernel<D>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+__device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
+                             int t, int wq, int lane, int q0, int h, int b) {
+  const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
+  const uint32_t tS = tmem + t * 128 + lane_off;
+  const uint32_t tO = tmem + 256 + t * 128 + lane_off;
+  const float sl2 = p.scale_log2;
+  float m_ref = -INFINITY;  // exp2-domain reference (scaled scores)
+  float l = 0.f;
+  bool ok = true;
+  for (int j = 0; j < p.total_tiles; ++j) {
+    int seg, tok0, valid;
+    tile_coord(p, j, seg, tok0, valid);
+    if (!(ok = wait_bar(&S->s_full[t], j & 1, S, p.status))) break;
+    tc_fence_after();
+    uint32_t s[4][32];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, s[c]);
+    tmem_wait_ld();
+    if (valid < kBN) {  // ragged end of a segment: mask the tail keys
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (c * 32 + i >= valid) s[c][i] = 0xff800000u;  // -inf
+    }
+    float mx = -INFINITY;
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+#pragma unroll
+      for (int i = 0; i < 32; ++i) mx = fmaxf(mx, __uint_as_float(s[c][i]));
+    mx *= sl2;
+    // Move the reference only when this tile's max passes it by more than
+    // the threshold (decided per warp: TMEM accesses are warp-wide).
+    float alpha = 1.f;
+    const bool rescale = __any_sync(0xffffffffu, mx > m_ref + kRescaleThreshold);
+    if (rescale) {
+      const float m_new = fmaxf(m_ref, mx);
+      alpha = ex2(m_ref - m_new);
+      l *= alpha;
+      m_ref = m_new;
+    }
+    const float neg = -m_ref;
+    float sum = 0.f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float p0 = ex2(fmaf(__uint_as_float(s[c][2 * i]), sl2, neg));
+        const float p1 = ex2(fmaf(__uint_as_float(s[c][2 * i + 1]), sl2, neg));
+        sum += p0 + p1;
+        pk[i] = pack_bf16(p0, p1);
+      }
+      tmem_st16(tS + c * 16, pk);
+    }
+    l += sum;
+    if (rescale && j > 0) {
+      // O_t holds PV_t(0..j-1) and PV_t(j) waits for p_full: scale in place.
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tO + c * 32, r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+        tmem_st32(tO + c * 32, r);
+      }
+    }
+    tmem_wait_st();
+    tc_fence_before();
+    mbar_arrive(&S->p_full[t]);
+  }
+  if (!ok || !wait_bar(&S->o_full, 0, S, p.status)) return;
+  tc_fence_after();
+  const int row = q0 + t * kBM + wq * 32 + lane;
+  const bool in_range = row < p.q_tokens;
+  const float inv_l = 1.f / l;
+  uint16_t* orow = p.o + (int64_t)b * p.o_str.batch +
+                   (int64_t)(in_range ? row : 0) * p.o_str.token +
+                   (int64_t)h * p.o_str.head;
+#pragma unroll
+  for (int c = 0; c < D / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(tO + c * 32, r);
+    tmem_wait_ld();
+    uint32_t pk[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      pk[i] = pack_bf16(__uint_as_float(r[2 * i]) * inv_l,
+                        __uint_as_float(r[2 * i + 1]) * inv_l);
+    if (in_range) {
+      uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+      for (int v = 0; v < 4; ++v)
+        dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+    }
+  }
+  if (p.lse != nullptr && in_range)
+    p.lse[((int64_t)b * p.heads + h) * p.q_tokens + row] =
+        (m_ref + __log2f(l)) * 0.6931471805599453f;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
+  using L = Layout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Shared* S = reinterpret_cast<Shared*>(smem + L::shared_off);
+  const int warp = threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  const int q0 = blockIdx.x * (kQTiles * kBM);
+  const int h = blockIdx.y, b = blockIdx.z;
+
+  if (warp == 9) {
+    tmem_alloc(&S->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  if (threadIdx.x == 256) {
+    mbar_init(&S->q_full, 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&S->k_full[s], 1);
+      mbar_init(&S->k_empty[s], 1);
+      mbar_init(&S->v_full[s], 1);
+      mbar_init(&S->v_empty[s], 1);
+    }
+    for (int t = 0; t < kQTiles; ++t) {
+      mbar_init(&S->s_full[t], 1);
+      mbar_init(&S->p_full[t], 4 * 32);
+    }
+    mbar_init(&S->o_full, 1);
+    mbar_init(&S->drain, 1);
+    S->abort = 0;
+    fence_barrier_init();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = S->tmem_base;
+
+  if (warp == 8) {
+    if (lane == 0) producer<D>(p, smem, S, q0, h, b);
+    __syncwarp();
+  } else if (warp == 9) {
+    if (lane == 0) mma_issuer<D>(p, smem, S, tmem);
+    __syncwarp();
+  } else {
+    softmax_role<D>(p, S, tmem, warp / 4, warp % 4, lane, q0, h, b);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ host
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType,
+                                  cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (fn == nullptr) {
+    cudaDriverEntryPointQueryResult q;
+    void* ptr = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// 4-D bf16 map over (x = d, token, head, batch) with a box of 64 x 128
+// (one 128-byte swizzled row per token); element strides in bytes.
+bool make_map(CUtensorMap* m, const void* base, int d, int64_t tokens,
+              int heads, int batch, int64_t token_stride_b,
+              int64_t head_stride_b, int64_t batch_stride_b) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  const cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)tokens,
+                              (cuuint64_t)heads, (cuuint64_t)batch};
+  const cuuint64_t strides[3] = {(cuuint64_t)token_stride_b,
+                                 (cuuint64_t)head_stride_b,
+                                 (cuuint64_t)batch_stride_b};
+  const cuuint32_t box[4] = {64, 128, 1, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base),
+             dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_d(const AttnParams& a, cudaStream_t stream) {
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  const int64_t es = 2;  // bytes per bf16
+  if (!make_map(&p.q_map, a.q, D, a.q_tokens, a.heads, a.batch,
+                a.q_str.token * es, a.q_str.head * es, a.q_str.batch * es))
+    return cudaErrorInvalidValue;
+  int tiles = 0;
+  for (int s = 0; s < kMaxSegments; ++s) {
+    const int src = s < a.num_segments ? s : 0;
+    // The map ends where the segment ends: keys past it read as zeros.
+    const int64_t end = a.seg_start[src] + a.seg_len[src];
+    if (!make_map(&p.k_map[s], a.k, D, end, a.heads, a.batch,
+                  a.kv_str.token * es, a.kv_str.head * es, a.kv_str.batch * es) ||
+        !make_map(&p.v_map[s], a.v, D, end, a.heads, a.batch,
+                  a.kv_str.token * es, a.kv_str.head * es, a.kv_str.batch * es))
+      return cudaErrorInvalidValue;
+    p.seg_start[s] = (int32_t)a.seg_start[src];
+    p.seg_len[s] = s < a.num_segments ? a.seg_len[s] : 0;
+    const int t = (p.seg_len[s] + kBN - 1) / kBN;
+    if (s == 0) p.seg_tiles0 = t;
+    tiles += t;
+  }
+  p.total_tiles = tiles;
+  p.o = a.o;
+  p.lse = a.lse;
+  p.o_str = a.q_str;
+  p.q_tokens = a.q_tokens;
+  p.heads = a.heads;
+  p.scale_log2 = a.scale_log2;
+  p.status = a.status;
+  const int smem = Layout<D>::bytes;
+  cudaError_t e = cudaFuncSetAttribute(
+      chunk_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((p.q_tokens + kBlockM - 1) / kBlockM, p.heads, p.batch);
-  chunk_attn_mma_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+  dim3 grid((a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM), a.heads,
+            a.batch);
+  chunk_attn_tc_kernel<D><<<grid, kThreads, smem, stream>>>(p);
   return cudaGetLastError();
 }
 
