@@ -149,6 +149,19 @@ FASTVR_API fastvr_status_t fastvr_plan_visible(fastvr_plan_t plan, int32_t* num_
                                     int64_t* seg_start, int64_t* seg_len,
                                     int64_t* visible_tokens);
 
+/* Failure-detection hook (tests).  stall != 0 makes the next attention
+ * launches of this plan wait, in the MMA-issuing thread, on a barrier that
+ * nothing arrives on; the kernel's bounded wait runs out after
+ * wait_limit_ns, every role stops, in-flight copies and MMAs are drained,
+ * tensor memory is released and FASTVR_ERR_TIMEOUT is recorded for
+ * fastvr_get_status.  The output of such a launch is undefined.  No GPU
+ * fault or hang results.  wait_limit_ns = 0 keeps the default limit
+ * (4 s per wait); stall = 0 with wait_limit_ns = 0 restores normal
+ * operation.  Host only.  Errors: INVALID_ARG. */
+FASTVR_API fastvr_status_t fastvr_debug_inject_stall(fastvr_plan_t plan,
+                                                     int32_t stall,
+                                                     uint64_t wait_limit_ns);
+
 /* Release a plan (host memory only; the cache stays the caller's). */
 FASTVR_API void fastvr_plan_destroy(fastvr_plan_t plan);
 

@@ -51,7 +51,7 @@ constexpr int kThreads = 320;   // 8 softmax warps + producer + MMA warp
 constexpr int kBox = 128 * 128; // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;      // log2 units
-constexpr uint64_t kWaitLimitNs = 4000000000ull;  // 4 s per wait
+constexpr uint64_t kDefaultWaitLimitNs = 4000000000ull;  // 4 s per wait
 
 struct TcParams {
   CUtensorMap q_map;                  // {d, Lq, H, B}
@@ -67,6 +67,8 @@ struct TcParams {
   int32_t total_tiles;
   float scale_log2;
   int* status;
+  uint64_t wait_limit_ns;
+  int32_t inject_stall;
 };
 
 struct Shared {
@@ -77,6 +79,7 @@ struct Shared {
   uint64_t o_full, drain;
   uint32_t tmem_base;
   int abort;
+  uint64_t wait_limit_ns;
 };
 
 template <int D>
@@ -113,7 +116,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*reinterpret_cast<volatile int*>(&S->abort)) return false;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
+    if (global_timer_ns() - t0 > S->wait_limit_ns) {
       *reinterpret_cast<volatile int*>(&S->abort) = 1;
       atomicExch(status, kDevTimeout);
       return false;
@@ -122,10 +125,11 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
 }
 
 // Bounded wait that ignores the abort flag (draining in-flight work).
-__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity,
+                                           const Shared* S) {
   const uint64_t t0 = global_timer_ns();
   while (!mbar_try_wait(bar, parity)) {
-    if (global_timer_ns() - t0 > kWaitLimitNs) return;
+    if (global_timer_ns() - t0 > S->wait_limit_ns) return;
   }
 }
 
@@ -172,11 +176,11 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S, int q0,
   }
   // Every issued load has landed before the CTA may exit (a no-op wait in
   // normal operation: consumers already waited for them).
-  drain_wait(&S->q_full, 0);
+  drain_wait(&S->q_full, 0, S);
   for (int i = max(0, nk - kStages); i < nk; ++i)
-    drain_wait(&S->k_full[i % kStages], (i / kStages) & 1);
+    drain_wait(&S->k_full[i % kStages], (i / kStages) & 1, S);
   for (int i = max(0, nv - kStages); i < nv; ++i)
-    drain_wait(&S->v_full[i % kStages], (i / kStages) & 1);
+    drain_wait(&S->v_full[i % kStages], (i / kStages) & 1, S);
 }
 
 template <int D>
@@ -212,8 +216,11 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     }
   };
 
-  bool ok = wait_bar(&S->q_full, 0, S, p.status) &&
-            wait_bar(&S->k_full[0], 0, S, p.status);
+  // Test hook: o_full receives no arrival before the end of the stream, so
+  // this wait runs out and exercises the abort path.
+  bool ok = !p.inject_stall || wait_bar(&S->o_full, 0, S, p.status);
+  ok = ok && wait_bar(&S->q_full, 0, S, p.status) &&
+       wait_bar(&S->k_full[0], 0, S, p.status);
   if (ok) {
     tc_fence_after();
     qk(0, 0);
@@ -250,7 +257,7 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   }
   if (ok) mma_commit(&S->o_full);
   mma_commit(&S->drain);
-  drain_wait(&S->drain, 0);
+  drain_wait(&S->drain, 0, S);
 }
 
 template <int D>
@@ -389,6 +396,7 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
+    S->wait_limit_ns = p.wait_limit_ns ? p.wait_limit_ns : kDefaultWaitLimitNs;
     fence_barrier_init();
   }
   tc_fence_before();
@@ -486,6 +494,8 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream) {
   p.heads = a.heads;
   p.scale_log2 = a.scale_log2;
   p.status = a.status;
+  p.wait_limit_ns = a.wait_limit_ns;
+  p.inject_stall = a.inject_stall;
   const int smem = Layout<D>::bytes;
   cudaError_t e = cudaFuncSetAttribute(
       chunk_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);

@@ -44,6 +44,8 @@ struct fastvr_plan_s {
   int32_t last_frames;   // frames of the newest chunk
   bool device_ready;
   int device;
+  int32_t inject_stall;    // failure-detection test hook
+  uint64_t wait_limit_ns;  // 0 = kernel default
 };
 
 namespace {
@@ -175,6 +177,8 @@ fastvr_status_t fastvr_attn_plan(const fastvr_attn_config_t* cfg,
   p->last_frames = 0;
   p->device_ready = false;
   p->device = -1;
+  p->inject_stall = 0;
+  p->wait_limit_ns = 0;
   *out = p;
   return FASTVR_OK;
 }
@@ -249,6 +253,8 @@ fastvr_status_t fastvr_chunk_attn_fwd(fastvr_plan_t p, const void* q, void* out,
   }
   a.scale_log2 = c.softmax_scale * 1.4426950408889634f;
   a.status = control_word(p);
+  a.wait_limit_ns = p->wait_limit_ns;
+  a.inject_stall = p->inject_stall;
   if (fastvr::launch_chunk_attn(a, reinterpret_cast<cudaStream_t>(stream)) !=
       cudaSuccess)
     return FASTVR_ERR_CUDA;
@@ -317,6 +323,14 @@ fastvr_status_t fastvr_plan_visible(fastvr_plan_t p, int32_t* num_segments,
   }
   *num_segments = (int32_t)segs.size();
   *visible_tokens = total;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_debug_inject_stall(fastvr_plan_t p, int32_t stall,
+                                          uint64_t wait_limit_ns) {
+  if (p == nullptr) return FASTVR_ERR_INVALID_ARG;
+  p->inject_stall = stall != 0;
+  p->wait_limit_ns = wait_limit_ns;
   return FASTVR_OK;
 }
 

@@ -49,6 +49,8 @@ struct AttnParams {
   int32_t seg_len[kMaxSegments];
   float scale_log2;       // softmax_scale * log2(e)
   int* status;            // control word (device)
+  uint64_t wait_limit_ns; // bound of every in-kernel wait (0 = default)
+  int32_t inject_stall;   // test hook: stall the MMA issuer until timeout
 };
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream);

@@ -56,6 +56,7 @@ SIGNATURES = {
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64)]),
+    "fastvr_debug_inject_stall": (_I32, [_VP, _I32, ctypes.c_uint64]),
     "fastvr_plan_destroy": (None, [_VP]),
     "fastvr_status_string": (ctypes.c_char_p, [_I32]),
 }
@@ -148,6 +149,12 @@ def fastvr_plan_visible(plan: int):
     _check(lib.fastvr_plan_visible(plan, ctypes.byref(n), st, ln,
                                    ctypes.byref(tot)), "fastvr_plan_visible")
     return [(st[i], ln[i]) for i in range(n.value)], tot.value
+
+
+def fastvr_debug_inject_stall(plan: int, stall: int,
+                              wait_limit_ns: int) -> None:
+    _check(lib.fastvr_debug_inject_stall(plan, stall, wait_limit_ns),
+           "fastvr_debug_inject_stall")
 
 
 def fastvr_plan_destroy(plan: int) -> None:
