@@ -9,8 +9,9 @@
 //
 // One CTA owns two 128-row query tiles of one (batch, head) and streams the
 // visible keys in 128-key tiles:
-//   warp 8      TMA producer: Q tiles once, then K and V tiles through
-//               two-stage rings (128-byte swizzled boxes of 64 columns).
+//   warp 8      TMA producer of the Q tiles (once) and the K ring (3 deep);
+//   warp 10     TMA producer of the V ring (2 deep); all tiles are
+//               128-byte swizzled boxes of 64 columns.
 //   warp 9      MMA issuer (one thread): S_t = Q_t K^T into TMEM, then
 //               O_t += P_t V with P_t read from TMEM.
 //   warps 0-3   softmax of query tile 0, one thread per row (TMEM lane);
@@ -46,8 +47,9 @@ using namespace sm100;
 constexpr int kBM = 128;        // query rows per tile (one TMEM lane each)
 constexpr int kBN = 128;        // keys per tile
 constexpr int kQTiles = 2;      // query tiles per CTA
-constexpr int kStages = 2;      // depth of the K and V rings
-constexpr int kThreads = 320;   // 8 softmax warps + producer + MMA warp
+constexpr int kKStages = 3;     // depth of the K ring
+constexpr int kVStages = 2;     // depth of the V ring
+constexpr int kThreads = 352;   // 8 softmax warps, K and V producers, MMA
 constexpr int kBox = 128 * 128; // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;      // log2 units
@@ -73,8 +75,8 @@ struct TcParams {
 
 struct Shared {
   uint64_t q_full;
-  uint64_t k_full[kStages], k_empty[kStages];
-  uint64_t v_full[kStages], v_empty[kStages];
+  uint64_t k_full[kKStages], k_empty[kKStages];
+  uint64_t v_full[kVStages], v_empty[kVStages];
   uint64_t s_full[kQTiles], p_full[kQTiles];
   uint64_t o_full, drain;
   uint32_t tmem_base;
@@ -90,9 +92,9 @@ struct Layout {
     return ((kQTiles + s) * kNB + bx) * kBox;
   }
   __host__ __device__ static constexpr int v(int s, int bx) {
-    return ((kQTiles + kStages + s) * kNB + bx) * kBox;
+    return ((kQTiles + kKStages + s) * kNB + bx) * kBox;
   }
-  static constexpr int shared_off = (kQTiles + 2 * kStages) * kNB * kBox;
+  static constexpr int shared_off = (kQTiles + kKStages + kVStages) * kNB * kBox;
   static constexpr int bytes = shared_off + 1024 /*Shared*/ + 1024 /*align*/;
 };
 
@@ -141,46 +143,45 @@ __device__ __forceinline__ void tile_coord(const TcParams& p, int j, int& seg,
   valid = min(kBN, p.seg_len[seg] - jj * kBN);
 }
 
-template <int D>
+// TMA producers, one thread each: the K producer also loads the query tiles.
+// K and V advance independently, so a slow V slot never holds back the next
+// K tile (QK^T of tile j+1 is issued before PV of tile j completes).
+template <int D, bool kIsK>
 __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S, int q0,
                          int h, int b) {
   using L = Layout<D>;
-  tma_prefetch_desc(&p.q_map);
-  for (int s = 0; s < kMaxSegments; ++s) {
-    tma_prefetch_desc(&p.k_map[s]);
-    tma_prefetch_desc(&p.v_map[s]);
+  constexpr int kStages = kIsK ? kKStages : kVStages;
+  uint64_t* full = kIsK ? S->k_full : S->v_full;
+  uint64_t* empty = kIsK ? S->k_empty : S->v_empty;
+  if (kIsK) {
+    tma_prefetch_desc(&p.q_map);
+    mbar_arrive_expect_tx(&S->q_full, kQTiles * L::kNB * kBox);
+    for (int t = 0; t < kQTiles; ++t)
+      for (int bx = 0; bx < L::kNB; ++bx)
+        tma_load_4d(&p.q_map, smem + L::q(t, bx), &S->q_full, bx * 64,
+                    q0 + t * kBM, h, b);
   }
-  mbar_arrive_expect_tx(&S->q_full, kQTiles * L::kNB * kBox);
-  for (int t = 0; t < kQTiles; ++t)
-    for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(&p.q_map, smem + L::q(t, bx), &S->q_full, bx * 64,
-                  q0 + t * kBM, h, b);
-  int nk = 0, nv = 0;
+  for (int s = 0; s < kMaxSegments; ++s)
+    tma_prefetch_desc(kIsK ? &p.k_map[s] : &p.v_map[s]);
+  int issued = 0;
   for (int j = 0; j < p.total_tiles; ++j) {
     const int st = j % kStages;
     const uint32_t ph = (j / kStages) & 1;
     int seg, tok0, valid;
     tile_coord(p, j, seg, tok0, valid);
-    if (!wait_bar(&S->k_empty[st], ph ^ 1, S, p.status)) break;
-    mbar_arrive_expect_tx(&S->k_full[st], L::kNB * kBox);
+    if (!wait_bar(&empty[st], ph ^ 1, S, p.status)) break;
+    mbar_arrive_expect_tx(&full[st], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(&p.k_map[seg], smem + L::k(st, bx), &S->k_full[st], bx * 64,
-                  tok0, h, b);
-    ++nk;
-    if (!wait_bar(&S->v_empty[st], ph ^ 1, S, p.status)) break;
-    mbar_arrive_expect_tx(&S->v_full[st], L::kNB * kBox);
-    for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(&p.v_map[seg], smem + L::v(st, bx), &S->v_full[st], bx * 64,
-                  tok0, h, b);
-    ++nv;
+      tma_load_4d(kIsK ? &p.k_map[seg] : &p.v_map[seg],
+                  smem + (kIsK ? L::k(st, bx) : L::v(st, bx)), &full[st],
+                  bx * 64, tok0, h, b);
+    ++issued;
   }
   // Every issued load has landed before the CTA may exit (a no-op wait in
   // normal operation: consumers already waited for them).
-  drain_wait(&S->q_full, 0, S);
-  for (int i = max(0, nk - kStages); i < nk; ++i)
-    drain_wait(&S->k_full[i % kStages], (i / kStages) & 1, S);
-  for (int i = max(0, nv - kStages); i < nv; ++i)
-    drain_wait(&S->v_full[i % kStages], (i / kStages) & 1, S);
+  if (kIsK) drain_wait(&S->q_full, 0, S);
+  for (int i = max(0, issued - kStages); i < issued; ++i)
+    drain_wait(&full[i % kStages], (i / kStages) & 1, S);
 }
 
 template <int D>
@@ -230,15 +231,15 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     mma_commit(&S->k_empty[0]);
   }
   for (int j = 0; ok && j < n; ++j) {
-    const int st = j % kStages;
-    const uint32_t ph = (j / kStages) & 1;
+    const int vs = j % kVStages;
+    const uint32_t vph = (j / kVStages) & 1;
     const int jn = j + 1;
-    const int stn = jn % kStages;
-    const uint32_t phn = (jn / kStages) & 1;
-    if (!(ok = wait_bar(&S->v_full[st], ph, S, p.status))) break;
+    const int stn = jn % kKStages;
+    const uint32_t phn = (jn / kKStages) & 1;
+    if (!(ok = wait_bar(&S->v_full[vs], vph, S, p.status))) break;
     if (!(ok = wait_bar(&S->p_full[0], j & 1, S, p.status))) break;
     tc_fence_after();
-    pv(0, st, j > 0);
+    pv(0, vs, j > 0);
     if (jn < n) {
       if (!(ok = wait_bar(&S->k_full[stn], phn, S, p.status))) break;
       tc_fence_after();
@@ -247,8 +248,8 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     }
     if (!(ok = wait_bar(&S->p_full[1], j & 1, S, p.status))) break;
     tc_fence_after();
-    pv(1, st, j > 0);
-    mma_commit(&S->v_empty[st]);
+    pv(1, vs, j > 0);
+    mma_commit(&S->v_empty[vs]);
     if (jn < n) {
       qk(1, stn);
       mma_commit(&S->s_full[1]);
@@ -260,6 +261,75 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   drain_wait(&S->drain, 0, S);
 }
 
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// P = 2^(s * scale_log2 - m) for the 32 columns of s[c] (a packed FFMA per
+// pair, one MUFU ex2 per element), stored as 16 bf16 pairs at TMEM column
+// tS + 16 c; the row sums go to four independent packed accumulators.
+__device__ __forceinline__ void exp_store32(const uint32_t (&sc)[32],
+                                            uint64_t sl2x2, uint64_t neg2,
+                                            uint32_t taddr, uint64_t (&acc)[4]) {
+  uint32_t pk[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const uint64_t x2 = f2_fma(f2_pack(__uint_as_float(sc[2 * i]),
+                                       __uint_as_float(sc[2 * i + 1])),
+                               sl2x2, neg2);
+    float x0, x1;
+    f2_unpack(x2, x0, x1);
+    const float p0 = ex2(x0), p1 = ex2(x1);
+    acc[i & 3] = f2_add(acc[i & 3], f2_pack(p0, p1));
+    pk[i] = pack_bf16(p0, p1);
+  }
+  tmem_st16(taddr, pk);
+}
+
+__device__ __forceinline__ float acc_total(const uint64_t (&acc)[4]) {
+  float a0, a1, b0, b1, c0, c1, d0, d1;
+  f2_unpack(acc[0], a0, a1);
+  f2_unpack(acc[1], b0, b1);
+  f2_unpack(acc[2], c0, c1);
+  f2_unpack(acc[3], d0, d1);
+  return ((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1));
+}
+
+// Mask columns >= valid of s[c] (the ragged end of a segment) and fold the
+// row max of s[c] into four independent accumulators.
+__device__ __forceinline__ void mask_max32(uint32_t (&sc)[32], int c, int valid,
+                                           float (&mx)[4]) {
+  if (valid < (c + 1) * 32) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (c * 32 + i >= valid) sc[i] = 0xff800000u;  // -inf
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    mx[i & 3] = max3(mx[i & 3], __uint_as_float(sc[2 * i]),
+                     __uint_as_float(sc[2 * i + 1]));
+}
+
 template <int D>
 __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
                              int t, int wq, int lane, int q0, int h, int b) {
@@ -267,6 +337,7 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   const uint32_t tS = tmem + t * 128 + lane_off;
   const uint32_t tO = tmem + 256 + t * 128 + lane_off;
   const float sl2 = p.scale_log2;
+  const uint64_t sl2x2 = f2_pack(sl2, sl2);
   float m_ref = -INFINITY;  // exp2-domain reference (scaled scores)
   float l = 0.f;
   bool ok = true;
@@ -276,47 +347,34 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     if (!(ok = wait_bar(&S->s_full[t], j & 1, S, p.status))) break;
     tc_fence_after();
     uint32_t s[4][32];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, s[c]);
+    tmem_ld32(tS + 0, s[0]);
+    tmem_ld32(tS + 32, s[1]);
     tmem_wait_ld();
-    if (valid < kBN) {  // ragged end of a segment: mask the tail keys
-#pragma unroll
-      for (int c = 0; c < 4; ++c)
-#pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (c * 32 + i >= valid) s[c][i] = 0xff800000u;  // -inf
-    }
-    float mx = -INFINITY;
-#pragma unroll
-    for (int c = 0; c < 4; ++c)
-#pragma unroll
-      for (int i = 0; i < 32; ++i) mx = fmaxf(mx, __uint_as_float(s[c][i]));
-    mx *= sl2;
-    // Move the reference only when this tile's max passes it by more than
-    // the threshold (decided per warp: TMEM accesses are warp-wide).
+    tmem_ld32(tS + 64, s[2]);  // lands while the first half is reduced
+    tmem_ld32(tS + 96, s[3]);
+    float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+    mask_max32(s[0], 0, valid, mx);
+    mask_max32(s[1], 1, valid, mx);
+    tmem_wait_ld();
+    mask_max32(s[2], 2, valid, mx);
+    mask_max32(s[3], 3, valid, mx);
+    const float mrow = fmaxf(max3(mx[0], mx[1], mx[2]), mx[3]) * sl2;
+    // The reference moves only when a row max passes it by more than the
+    // threshold (decided per warp: TMEM accesses are warp-wide).
+    const bool rescale =
+        __any_sync(0xffffffffu, mrow > m_ref + kRescaleThreshold);
     float alpha = 1.f;
-    const bool rescale = __any_sync(0xffffffffu, mx > m_ref + kRescaleThreshold);
     if (rescale) {
-      const float m_new = fmaxf(m_ref, mx);
+      const float m_new = fmaxf(m_ref, mrow);
       alpha = ex2(m_ref - m_new);
       l *= alpha;
       m_ref = m_new;
     }
-    const float neg = -m_ref;
-    float sum = 0.f;
+    const uint64_t neg2 = f2_pack(-m_ref, -m_ref);
+    uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      uint32_t pk[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float p0 = ex2(fmaf(__uint_as_float(s[c][2 * i]), sl2, neg));
-        const float p1 = ex2(fmaf(__uint_as_float(s[c][2 * i + 1]), sl2, neg));
-        sum += p0 + p1;
-        pk[i] = pack_bf16(p0, p1);
-      }
-      tmem_st16(tS + c * 16, pk);
-    }
-    l += sum;
+    for (int c = 0; c < 4; ++c) exp_store32(s[c], sl2x2, neg2, tS + 16 * c, acc);
+    l += acc_total(acc);
     if (rescale && j > 0) {
       // O_t holds PV_t(0..j-1) and PV_t(j) waits for p_full: scale in place.
 #pragma unroll
@@ -383,9 +441,11 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   }
   if (threadIdx.x == 256) {
     mbar_init(&S->q_full, 1);
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kKStages; ++s) {
       mbar_init(&S->k_full[s], 1);
       mbar_init(&S->k_empty[s], 1);
+    }
+    for (int s = 0; s < kVStages; ++s) {
       mbar_init(&S->v_full[s], 1);
       mbar_init(&S->v_empty[s], 1);
     }
@@ -405,7 +465,10 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   const uint32_t tmem = S->tmem_base;
 
   if (warp == 8) {
-    if (lane == 0) producer<D>(p, smem, S, q0, h, b);
+    if (lane == 0) producer<D, true>(p, smem, S, q0, h, b);
+    __syncwarp();
+  } else if (warp == 10) {
+    if (lane == 0) producer<D, false>(p, smem, S, q0, h, b);
     __syncwarp();
   } else if (warp == 9) {
     if (lane == 0) mma_issuer<D>(p, smem, S, tmem);
