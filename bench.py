@@ -268,12 +268,14 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
         time.sleep(0.3)
     barrier(world)
     torch.cuda.synchronize(dev)
+    launches_before = att.launch_count()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
     for s in range(args.steps):
         step(evs[s])
     t_end.record(stream)
+    launches = att.launch_count() - launches_before
     torch.cuda.synchronize(dev)
     barrier(world)
     clock_info = clocks.stop() if clocks else None
@@ -331,7 +333,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
                      "peak_kind": f"{peak_kind} bf16 sustained",
                      "kernel": "chunk_attn_fwd",
                      "traffic": traffic},
-        "gpu_launches": 2 * w.num_chunks * args.steps,
+        "gpu_launches": launches,
         "clocks": clock_info,
         "e2e": e2e,
     }

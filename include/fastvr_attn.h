@@ -81,8 +81,9 @@ typedef struct fastvr_plan_s* fastvr_plan_t;
 
 /* Bytes of device memory the caller must provide for the KV cache of cfg:
  * K and V, each [B, H, S*k*N, d] bfloat16 with S = window_chunks + 1 slots
- * (bounded window) or max_chunks slots (unbounded), plus a 256-byte control
- * block at the end.  Host only; no device work.
+ * (bounded window) or max_chunks slots (unbounded), then the attention
+ * kernel's split-KV workspace (256 x 256 x (d + 1) floats), then a 256-byte
+ * control block.  Host only; no device work.
  * Errors: INVALID_ARG (null, non-positive sizes), UNSUPPORTED (head_dim). */
 FASTVR_API fastvr_status_t fastvr_kv_cache_bytes(const fastvr_attn_config_t* cfg,
                                       size_t* bytes);
@@ -148,6 +149,12 @@ FASTVR_API fastvr_status_t fastvr_plan_set_state(fastvr_plan_t plan, int64_t chu
 FASTVR_API fastvr_status_t fastvr_plan_visible(fastvr_plan_t plan, int32_t* num_segments,
                                     int64_t* seg_start, int64_t* seg_len,
                                     int64_t* visible_tokens);
+
+/* Number of kernel launches this plan has enqueued since it was created
+ * (an append is one launch; an attention call is one, or two when the key
+ * range of some query units is split across SMs and merged).  Host only. */
+FASTVR_API fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t plan,
+                                                    int64_t* launches);
 
 /* Failure-detection hook (tests).  stall != 0 makes the next attention
  * launches of this plan wait, in the MMA-issuing thread, on a barrier that

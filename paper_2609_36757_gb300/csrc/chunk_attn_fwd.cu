@@ -36,6 +36,8 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include <algorithm>
+
 #include "fastvr_internal.h"
 #include "sm100_ptx.cuh"
 
@@ -53,6 +55,7 @@ constexpr int kThreads = 352;   // 8 softmax warps, K and V producers, MMA
 constexpr int kBox = 128 * 128; // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;      // log2 units
+constexpr int kMinTilesPerPart = 4;             // key tiles per split part
 constexpr uint64_t kDefaultWaitLimitNs = 4000000000ull;  // 4 s per wait
 
 struct TcParams {
@@ -71,7 +74,43 @@ struct TcParams {
   int* status;
   uint64_t wait_limit_ns;
   int32_t inject_stall;
+  // Work split: units of two query tiles, (b, h, pair) with the pair index
+  // fastest; the first units_full run whole, the rest are cut into `split`
+  // key-tile ranges whose partial results go to the workspace.
+  int32_t q_pairs, units_full, split;
+  float* ws;
 };
+
+// The work of one CTA.
+struct Work {
+  int q0, h, b;
+  int j0, n;   // first key tile (index into the visible tiles) and count
+  int nqt;     // query tiles with at least one row in the chunk (1 or 2)
+  int part;    // -1: whole unit, final output; else workspace slot
+};
+
+__device__ __forceinline__ Work cta_work(const TcParams& p) {
+  Work w;
+  int unit, part = -1, nparts = 1, idx = 0;
+  if ((int)blockIdx.x < p.units_full) {
+    unit = blockIdx.x;
+  } else {
+    const int k = blockIdx.x - p.units_full;
+    unit = p.units_full + k / p.split;
+    idx = k % p.split;
+    part = k;
+    nparts = p.split;
+  }
+  const int pair = unit % p.q_pairs;
+  w.h = (unit / p.q_pairs) % p.heads;
+  w.b = unit / (p.q_pairs * p.heads);
+  w.q0 = pair * kQTiles * kBM;
+  w.nqt = (p.q_tokens - w.q0 > kBM) ? 2 : 1;
+  w.j0 = (int)((int64_t)idx * p.total_tiles / nparts);
+  w.n = (int)((int64_t)(idx + 1) * p.total_tiles / nparts) - w.j0;
+  w.part = part;
+  return w;
+}
 
 struct Shared {
   uint64_t q_full;
@@ -147,28 +186,29 @@ __device__ __forceinline__ void tile_coord(const TcParams& p, int j, int& seg,
 // K and V advance independently, so a slow V slot never holds back the next
 // K tile (QK^T of tile j+1 is issued before PV of tile j completes).
 template <int D, bool kIsK>
-__device__ void producer(const TcParams& p, uint8_t* smem, Shared* S, int q0,
-                         int h, int b) {
+__device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
+                         const Work& w) {
+  const int h = w.h, b = w.b;
   using L = Layout<D>;
   constexpr int kStages = kIsK ? kKStages : kVStages;
   uint64_t* full = kIsK ? S->k_full : S->v_full;
   uint64_t* empty = kIsK ? S->k_empty : S->v_empty;
   if (kIsK) {
     tma_prefetch_desc(&p.q_map);
-    mbar_arrive_expect_tx(&S->q_full, kQTiles * L::kNB * kBox);
-    for (int t = 0; t < kQTiles; ++t)
+    mbar_arrive_expect_tx(&S->q_full, w.nqt * L::kNB * kBox);
+    for (int t = 0; t < w.nqt; ++t)
       for (int bx = 0; bx < L::kNB; ++bx)
         tma_load_4d(&p.q_map, smem + L::q(t, bx), &S->q_full, bx * 64,
-                    q0 + t * kBM, h, b);
+                    w.q0 + t * kBM, h, b);
   }
   for (int s = 0; s < kMaxSegments; ++s)
     tma_prefetch_desc(kIsK ? &p.k_map[s] : &p.v_map[s]);
   int issued = 0;
-  for (int j = 0; j < p.total_tiles; ++j) {
+  for (int j = 0; j < w.n; ++j) {
     const int st = j % kStages;
     const uint32_t ph = (j / kStages) & 1;
     int seg, tok0, valid;
-    tile_coord(p, j, seg, tok0, valid);
+    tile_coord(p, w.j0 + j, seg, tok0, valid);
     if (!wait_bar(&empty[st], ph ^ 1, S, p.status)) break;
     mbar_arrive_expect_tx(&full[st], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
@@ -186,12 +226,13 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S, int q0,
 
 template <int D>
 __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
-                           uint32_t tmem) {
+                           uint32_t tmem, const Work& w) {
   using L = Layout<D>;
   constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, 0);
   constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, D, 1);
   const uint32_t sbase = smem_addr(smem);
-  const int n = p.total_tiles;
+  const int n = w.n;
+  const bool two = w.nqt == 2;
 
   // S_t = Q_t K^T: both operands K-major, 128-byte swizzle; a K step of 16
   // elements is 32 bytes inside a 64-column box.
@@ -226,8 +267,10 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     tc_fence_after();
     qk(0, 0);
     mma_commit(&S->s_full[0]);
-    qk(1, 0);
-    mma_commit(&S->s_full[1]);
+    if (two) {
+      qk(1, 0);
+      mma_commit(&S->s_full[1]);
+    }
     mma_commit(&S->k_empty[0]);
   }
   for (int j = 0; ok && j < n; ++j) {
@@ -246,13 +289,17 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
       qk(0, stn);
       mma_commit(&S->s_full[0]);
     }
-    if (!(ok = wait_bar(&S->p_full[1], j & 1, S, p.status))) break;
-    tc_fence_after();
-    pv(1, vs, j > 0);
+    if (two) {
+      if (!(ok = wait_bar(&S->p_full[1], j & 1, S, p.status))) break;
+      tc_fence_after();
+      pv(1, vs, j > 0);
+    }
     mma_commit(&S->v_empty[vs]);
     if (jn < n) {
-      qk(1, stn);
-      mma_commit(&S->s_full[1]);
+      if (two) {
+        qk(1, stn);
+        mma_commit(&S->s_full[1]);
+      }
       mma_commit(&S->k_empty[stn]);
     }
   }
@@ -332,7 +379,7 @@ __device__ __forceinline__ void mask_max32(uint32_t (&sc)[32], int c, int valid,
 
 template <int D>
 __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
-                             int t, int wq, int lane, int q0, int h, int b) {
+                             int t, int wq, int lane, int j0, int n) {
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
   const uint32_t tS = tmem + t * 128 + lane_off;
   const uint32_t tO = tmem + 256 + t * 128 + lane_off;
@@ -341,9 +388,9 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   float m_ref = -INFINITY;  // exp2-domain reference (scaled scores)
   float l = 0.f;
   bool ok = true;
-  for (int j = 0; j < p.total_tiles; ++j) {
+  for (int j = 0; j < n; ++j) {
     int seg, tok0, valid;
-    tile_coord(p, j, seg, tok0, valid);
+    tile_coord(p, j0 + j, seg, tok0, valid);
     if (!(ok = wait_bar(&S->s_full[t], j & 1, S, p.status))) break;
     tc_fence_after();
     uint32_t s[4][32];
@@ -394,12 +441,32 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   }
   if (!ok || !wait_bar(&S->o_full, 0, S, p.status)) return;
   tc_fence_after();
-  const int row = q0 + t * kBM + wq * 32 + lane;
-  const bool in_range = row < p.q_tokens;
+  const Work w = cta_work(p);
+  const int r_unit = t * kBM + wq * 32 + lane;  // row within the unit
+  const int row = w.q0 + r_unit;
   const float inv_l = 1.f / l;
-  uint16_t* orow = p.o + (int64_t)b * p.o_str.batch +
+  if (w.part >= 0) {
+    // Partial result of a key range: O / l in fp32 (transposed, so a warp's
+    // stores are contiguous) and the log2-domain log-sum-exp.
+    float* ws_o = p.ws + (size_t)w.part * D * kUnitRows;
+    float* ws_l = p.ws + (size_t)kMaxParts * D * kUnitRows +
+                  (size_t)w.part * kUnitRows;
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t r[32];
+      tmem_ld32(tO + c * 32, r);
+      tmem_wait_ld();
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        ws_o[(c * 32 + i) * kUnitRows + r_unit] = __uint_as_float(r[i]) * inv_l;
+    }
+    ws_l[r_unit] = m_ref + __log2f(l);
+    return;
+  }
+  const bool in_range = row < p.q_tokens;
+  uint16_t* orow = p.o + (int64_t)w.b * p.o_str.batch +
                    (int64_t)(in_range ? row : 0) * p.o_str.token +
-                   (int64_t)h * p.o_str.head;
+                   (int64_t)w.h * p.o_str.head;
 #pragma unroll
   for (int c = 0; c < D / 32; ++c) {
     uint32_t r[32];
@@ -418,8 +485,59 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     }
   }
   if (p.lse != nullptr && in_range)
-    p.lse[((int64_t)b * p.heads + h) * p.q_tokens + row] =
+    p.lse[((int64_t)w.b * p.heads + w.h) * p.q_tokens + row] =
         (m_ref + __log2f(l)) * 0.6931471805599453f;
+}
+
+// Merge the partial results of the split units: weights 2^(lse_i - m),
+// O = sum_i w_i O_i / sum_i w_i, LSE = m + log2(sum_i w_i) (natural log out).
+// One thread per query row, 128 rows per CTA; workspace reads are coalesced.
+template <int D>
+__global__ void __launch_bounds__(128)
+combine_kernel(const __grid_constant__ TcParams p) {
+  const int ut = blockIdx.x;
+  const int r_unit = blockIdx.y * 128 + threadIdx.x;
+  const int unit = p.units_full + ut;
+  const int pair = unit % p.q_pairs;
+  const int h = (unit / p.q_pairs) % p.heads;
+  const int b = unit / (p.q_pairs * p.heads);
+  const int row = pair * kQTiles * kBM + r_unit;
+  if (row >= p.q_tokens) return;
+  const int k0 = ut * p.split;
+  const float* ws_l = p.ws + (size_t)kMaxParts * D * kUnitRows;
+  float m = -INFINITY;
+  for (int i = 0; i < p.split; ++i)
+    m = fmaxf(m, ws_l[(size_t)(k0 + i) * kUnitRows + r_unit]);
+  float wsum = 0.f;
+  for (int i = 0; i < p.split; ++i)
+    wsum += ex2(ws_l[(size_t)(k0 + i) * kUnitRows + r_unit] - m);
+  const float inv = 1.f / wsum;
+  uint16_t* orow = p.o + (int64_t)b * p.o_str.batch +
+                   (int64_t)row * p.o_str.token + (int64_t)h * p.o_str.head;
+#pragma unroll 1
+  for (int c = 0; c < D / 32; ++c) {
+    float acc[32];
+#pragma unroll
+    for (int x = 0; x < 32; ++x) acc[x] = 0.f;
+    for (int i = 0; i < p.split; ++i) {
+      const float wi =
+          ex2(ws_l[(size_t)(k0 + i) * kUnitRows + r_unit] - m) * inv;
+      const float* src =
+          p.ws + ((size_t)(k0 + i) * D + c * 32) * kUnitRows + r_unit;
+#pragma unroll
+      for (int x = 0; x < 32; ++x) acc[x] = fmaf(wi, src[x * kUnitRows], acc[x]);
+    }
+    uint32_t pk[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) pk[i] = pack_bf16(acc[2 * i], acc[2 * i + 1]);
+    uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+    for (int v = 0; v < 4; ++v)
+      dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+  }
+  if (p.lse != nullptr)
+    p.lse[((int64_t)b * p.heads + h) * p.q_tokens + row] =
+        (m + __log2f(wsum)) * 0.6931471805599453f;
 }
 
 template <int D>
@@ -432,8 +550,7 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   Shared* S = reinterpret_cast<Shared*>(smem + L::shared_off);
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
-  const int q0 = blockIdx.x * (kQTiles * kBM);
-  const int h = blockIdx.y, b = blockIdx.z;
+  const Work w = cta_work(p);
 
   if (warp == 9) {
     tmem_alloc(&S->tmem_base, kTmemCols);
@@ -465,16 +582,18 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   const uint32_t tmem = S->tmem_base;
 
   if (warp == 8) {
-    if (lane == 0) producer<D, true>(p, smem, S, q0, h, b);
+    if (lane == 0) producer<D, true>(p, smem, S, w);
     __syncwarp();
   } else if (warp == 10) {
-    if (lane == 0) producer<D, false>(p, smem, S, q0, h, b);
+    if (lane == 0) producer<D, false>(p, smem, S, w);
     __syncwarp();
   } else if (warp == 9) {
-    if (lane == 0) mma_issuer<D>(p, smem, S, tmem);
+    if (lane == 0) mma_issuer<D>(p, smem, S, tmem, w);
     __syncwarp();
   } else {
-    softmax_role<D>(p, S, tmem, warp / 4, warp % 4, lane, q0, h, b);
+    // A query tile that lies past the end of the chunk has no work.
+    if (warp / 4 < w.nqt)
+      softmax_role<D>(p, S, tmem, warp / 4, warp % 4, lane, w.j0, w.n);
   }
   tc_fence_before();
   __syncthreads();
@@ -507,6 +626,13 @@ EncodeTiledFn encode_fn() {
 
 // 4-D bf16 map over (x = d, token, head, batch) with a box of 64 x 128
 // (one 128-byte swizzled row per token); element strides in bytes.
+int sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
 bool make_map(CUtensorMap* m, const void* base, int d, int64_t tokens,
               int heads, int batch, int64_t token_stride_b,
               int64_t head_stride_b, int64_t batch_stride_b) {
@@ -526,7 +652,7 @@ bool make_map(CUtensorMap* m, const void* base, int d, int64_t tokens,
 }
 
 template <int D>
-cudaError_t launch_d(const AttnParams& a, cudaStream_t stream) {
+cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
   TcParams p;
   memset(&p, 0, sizeof(p));
   const int64_t es = 2;  // bytes per bf16
@@ -559,21 +685,48 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream) {
   p.status = a.status;
   p.wait_limit_ns = a.wait_limit_ns;
   p.inject_stall = a.inject_stall;
+  p.ws = a.workspace;
+
+  // Units of two query tiles; whole waves of units run whole, and the units
+  // of a last partial wave are cut along the keys so that every SM has work
+  // (at least kMinTilesPerPart key tiles per part).
+  const int sms = sm_count();
+  p.q_pairs = (a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);
+  const int units = p.q_pairs * a.heads * a.batch;
+  const int rem = units % sms;
+  int split = 1;
+  if (rem > 0) {
+    split = std::min(sms / rem, tiles / kMinTilesPerPart);
+    split = std::min(split, kMaxParts / rem);
+  }
+  if (split >= 2) {
+    p.units_full = units - rem;
+    p.split = split;
+  } else {
+    p.units_full = units;
+    p.split = 1;
+  }
+  const int grid = p.units_full + (units - p.units_full) * p.split;
   const int smem = Layout<D>::bytes;
   cudaError_t e = cudaFuncSetAttribute(
       chunk_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM), a.heads,
-            a.batch);
   chunk_attn_tc_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+  *launches = 1;
+  if (p.split > 1) {
+    combine_kernel<D><<<dim3(units - p.units_full, kQTiles), 128, 0, stream>>>(p);
+    *launches = 2;
+  }
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream) {
-  if (p.head_dim == 64) return launch_d<64>(p, stream);
-  if (p.head_dim == 128) return launch_d<128>(p, stream);
+cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream,
+                              int* launches) {
+  *launches = 0;
+  if (p.head_dim == 64) return launch_d<64>(p, stream, launches);
+  if (p.head_dim == 128) return launch_d<128>(p, stream, launches);
   return cudaErrorInvalidValue;
 }
 

@@ -44,6 +44,7 @@ struct fastvr_plan_s {
   int32_t last_frames;   // frames of the newest chunk
   bool device_ready;
   int device;
+  int64_t launches;        // kernels enqueued since creation
   int32_t inject_stall;    // failure-detection test hook
   uint64_t wait_limit_ns;  // 0 = kernel default
 };
@@ -89,6 +90,15 @@ std::vector<Segment> visible_segments(const fastvr_plan_s& p) {
   return segs;
 }
 
+float* workspace(const fastvr_plan_s* p) {
+  return reinterpret_cast<float*>(p->base + 2 * p->kv_bytes);
+}
+
+int* control_word(const fastvr_plan_s* p) {
+  return reinterpret_cast<int*>(p->base + 2 * p->kv_bytes +
+                                fastvr::workspace_bytes(p->cfg.head_dim));
+}
+
 fastvr_status_t ensure_device(fastvr_plan_s* p) {
   if (p->device_ready) return FASTVR_OK;
   int dev = 0;
@@ -107,15 +117,11 @@ fastvr_status_t ensure_device(fastvr_plan_s* p) {
     return FASTVR_ERR_INVALID_ARG;
   }
   // Clear the control block once; kernels only ever set it.
-  if (cudaMemset(p->base + 2 * p->kv_bytes, 0, kControlBytes) != cudaSuccess)
+  if (cudaMemset(control_word(p), 0, kControlBytes) != cudaSuccess)
     return FASTVR_ERR_CUDA;
   p->device = dev;
   p->device_ready = true;
   return FASTVR_OK;
-}
-
-int* control_word(const fastvr_plan_s* p) {
-  return reinterpret_cast<int*>(p->base + 2 * p->kv_bytes);
 }
 
 }  // namespace
@@ -145,7 +151,8 @@ fastvr_status_t fastvr_kv_cache_bytes(const fastvr_attn_config_t* cfg,
   // K and V regions, each a multiple of 256 bytes (d*2 >= 128 and tokens of
   // a slot are whole rows, so per is a multiple of 128; round up anyway).
   const int64_t region = (per + 255) / 256 * 256;
-  *bytes = (size_t)(2 * region) + kControlBytes;
+  *bytes = (size_t)(2 * region) + fastvr::workspace_bytes(cfg->head_dim) +
+           kControlBytes;
   return FASTVR_OK;
 }
 
@@ -171,12 +178,14 @@ fastvr_status_t fastvr_attn_plan(const fastvr_attn_config_t* cfg,
   p->slots = num_slots(*cfg);
   p->slot_tokens = (int64_t)cfg->frames_per_chunk * cfg->tokens_per_frame;
   p->cache_tokens = p->slots * p->slot_tokens;
-  p->kv_bytes = (need - kControlBytes) / 2;
+  p->kv_bytes =
+      (need - kControlBytes - fastvr::workspace_bytes(cfg->head_dim)) / 2;
   p->base = static_cast<char*>(kv_cache);
   p->chunks = 0;
   p->last_frames = 0;
   p->device_ready = false;
   p->device = -1;
+  p->launches = 0;
   p->inject_stall = 0;
   p->wait_limit_ns = 0;
   *out = p;
@@ -211,6 +220,7 @@ fastvr_status_t fastvr_kv_append(fastvr_plan_t p, const void* k_new,
   if (fastvr::launch_kv_append(a, reinterpret_cast<cudaStream_t>(stream)) !=
       cudaSuccess)
     return FASTVR_ERR_CUDA;
+  p->launches += 1;
   p->chunks += 1;
   p->last_frames = frames;
   return FASTVR_OK;
@@ -253,11 +263,14 @@ fastvr_status_t fastvr_chunk_attn_fwd(fastvr_plan_t p, const void* q, void* out,
   }
   a.scale_log2 = c.softmax_scale * 1.4426950408889634f;
   a.status = control_word(p);
+  a.workspace = workspace(p);
   a.wait_limit_ns = p->wait_limit_ns;
   a.inject_stall = p->inject_stall;
-  if (fastvr::launch_chunk_attn(a, reinterpret_cast<cudaStream_t>(stream)) !=
-      cudaSuccess)
-    return FASTVR_ERR_CUDA;
+  int launched = 0;
+  const cudaError_t e = fastvr::launch_chunk_attn(
+      a, reinterpret_cast<cudaStream_t>(stream), &launched);
+  p->launches += launched;
+  if (e != cudaSuccess) return FASTVR_ERR_CUDA;
   return FASTVR_OK;
 }
 
@@ -323,6 +336,12 @@ fastvr_status_t fastvr_plan_visible(fastvr_plan_t p, int32_t* num_segments,
   }
   *num_segments = (int32_t)segs.size();
   *visible_tokens = total;
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t p, int64_t* launches) {
+  if (p == nullptr || launches == nullptr) return FASTVR_ERR_INVALID_ARG;
+  *launches = p->launches;
   return FASTVR_OK;
 }
 

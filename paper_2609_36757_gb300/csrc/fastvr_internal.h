@@ -13,6 +13,14 @@ namespace fastvr {
 // Sec. 3.1 KV caching).
 constexpr int kMaxSegments = 2;
 
+// Split-KV workspace of the attention kernel: at most kMaxParts partial
+// results of 256 query rows, each d fp32 outputs plus one log-sum-exp.
+constexpr int kMaxParts = 256;
+constexpr int kUnitRows = 256;
+inline size_t workspace_bytes(int head_dim) {
+  return (size_t)kMaxParts * kUnitRows * (head_dim + 1) * sizeof(float);
+}
+
 // Error codes a kernel writes into the cache's control block.
 constexpr int kDevOk = 0;
 constexpr int kDevTimeout = 1;
@@ -49,11 +57,15 @@ struct AttnParams {
   int32_t seg_len[kMaxSegments];
   float scale_log2;       // softmax_scale * log2(e)
   int* status;            // control word (device)
+  float* workspace;       // workspace_bytes(head_dim) of scratch (device)
   uint64_t wait_limit_ns; // bound of every in-kernel wait (0 = default)
   int32_t inject_stall;   // test hook: stall the MMA issuer until timeout
 };
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream);
-cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream);
+// Enqueues the attention kernel (and the merge kernel when the key range of
+// some units is split); *launches receives the number of kernels enqueued.
+cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream,
+                              int* launches);
 
 }  // namespace fastvr

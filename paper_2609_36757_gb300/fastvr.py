@@ -56,6 +56,7 @@ SIGNATURES = {
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64)]),
+    "fastvr_plan_launch_count": (_I32, [_VP, ctypes.POINTER(_I64)]),
     "fastvr_debug_inject_stall": (_I32, [_VP, _I32, ctypes.c_uint64]),
     "fastvr_plan_destroy": (None, [_VP]),
     "fastvr_status_string": (ctypes.c_char_p, [_I32]),
@@ -151,6 +152,13 @@ def fastvr_plan_visible(plan: int):
     return [(st[i], ln[i]) for i in range(n.value)], tot.value
 
 
+def fastvr_plan_launch_count(plan: int) -> int:
+    n = _I64(0)
+    _check(lib.fastvr_plan_launch_count(plan, ctypes.byref(n)),
+           "fastvr_plan_launch_count")
+    return n.value
+
+
 def fastvr_debug_inject_stall(plan: int, stall: int,
                               wait_limit_ns: int) -> None:
     _check(lib.fastvr_debug_inject_stall(plan, stall, wait_limit_ns),
@@ -229,6 +237,9 @@ class StreamingAttention:
 
     def reset(self) -> None:
         fastvr_plan_reset(self.plan)
+
+    def launch_count(self) -> int:
+        return fastvr_plan_launch_count(self.plan)
 
     def status(self) -> int:
         return fastvr_get_status(self.plan)

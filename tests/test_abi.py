@@ -49,12 +49,19 @@ def test_status_strings(fv):
 
 
 def test_cache_bytes_formula(fv):
+    # K and V regions, the split-KV workspace (256 parts x 256 rows x
+    # (d + 1) floats), the 256-byte control block
+    ws = lambda d: 256 * 256 * (d + 1) * 4
     cfg = fv.make_config(2, 3, 128, 10, 3, window_chunks=4)
     slots = 5
     per = 2 * 3 * slots * 3 * 10 * 128 * 2
-    assert fv.fastvr_kv_cache_bytes(cfg) == 2 * ((per + 255) // 256 * 256) + 256
+    assert fv.fastvr_kv_cache_bytes(cfg) == \
+        2 * ((per + 255) // 256 * 256) + ws(128) + 256
     cfg = fv.make_config(1, 12, 128, 8160, 2, -1, 15)
-    assert fv.fastvr_kv_cache_bytes(cfg) == 2 * 12 * 15 * 2 * 8160 * 256 + 256
+    assert fv.fastvr_kv_cache_bytes(cfg) == \
+        2 * 12 * 15 * 2 * 8160 * 256 + ws(128) + 256
+    cfg = fv.make_config(1, 2, 64, 64, 2, -1, 3)
+    assert fv.fastvr_kv_cache_bytes(cfg) == 2 * 2 * 3 * 2 * 64 * 128 + ws(64) + 256
 
 
 @pytest.mark.parametrize("kw,code", [

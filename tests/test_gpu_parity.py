@@ -69,6 +69,13 @@ SMALL = [
     WL.custom("ring-wrap", batch=1, heads=2, head_dim=128, tokens_per_frame=64,
               frames_per_chunk=2, num_chunks=9, window_chunks=3,
               last_chunk_frames=1, seed=27),
+    # few query units, long key ranges: the units are cut into many key
+    # ranges whose partial results are merged
+    WL.custom("split-many", batch=1, heads=1, head_dim=128,
+              tokens_per_frame=256, frames_per_chunk=2, num_chunks=8, seed=28),
+    WL.custom("split-d64-ragged", batch=1, heads=1, head_dim=64,
+              tokens_per_frame=200, frames_per_chunk=3, num_chunks=7,
+              window_chunks=5, last_chunk_frames=1, seed=29),
 ]
 
 
