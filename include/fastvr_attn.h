@@ -150,6 +150,43 @@ FASTVR_API fastvr_status_t fastvr_plan_visible(fastvr_plan_t plan, int32_t* num_
                                     int64_t* seg_start, int64_t* seg_len,
                                     int64_t* visible_tokens);
 
+/* Chunk-causal attention that allocates nothing (no counterpart in the
+ * paper; an interface for callers that cannot allocate device memory).
+ * Callers such as serving runtimes that own all device memory through their
+ * own pool, or real-time pipelines that forbid cudaMalloc/cudaFree after
+ * start-up because those calls can synchronise the device, keep K and V in
+ * their own buffers and cannot give the library the workspace region of
+ * fastvr_kv_cache_bytes.  This entry point needs neither a plan nor that
+ * region: its scratch (the partial results of query units whose key range
+ * is split across SMs, and a status word) is a fixed 24 MiB array in device
+ * memory, part of the library image, which every GPU that loads the library
+ * holds until the process exits.
+ *   q        bf16 [B, q_frames*N, H, d] token-major (cfg: B, H, d, N, scale;
+ *            frames_per_chunk, window_chunks and max_chunks are not used)
+ *   k_cache, v_cache  bf16 [B, H, cache_tokens, d] head-major (any buffers
+ *            of the caller, e.g. a plan's cache regions)
+ *   num_segments (1..2), seg_start, seg_len: the visible key ranges of one
+ *            head's cache, as fastvr_plan_visible reports them
+ *   out      bf16 [B, q_frames*N, H, d]; lse nullable, float32 [B, H, Lq]
+ * The result equals fastvr_chunk_attn_fwd's for the same inputs (same
+ * kernels, same work split).  The first call on each device resolves the
+ * array's device address (a symbol lookup, no allocation): make that first
+ * call before any stream capture.  Every call on a device shares the array
+ * and it keeps the last call's contents (each call clears the status word
+ * first), so calls that overlap on the GPU (other streams, other threads)
+ * race: serialise them.  A bounded-wait timeout leaves out undefined and is
+ * not reported.  No cudaMalloc, cudaFree or allocating library routine is
+ * called.
+ * Errors: INVALID_ARG (null or misaligned pointers, bad sizes or ranges),
+ * UNSUPPORTED (head_dim, device not sm_103), CAPACITY (the call's split
+ * needs more partial results than the array holds: 190 at d = 128, 378 at
+ * d = 64), CUDA. */
+FASTVR_API fastvr_status_t fastvr_chunk_attn_fwd_static(
+    const fastvr_attn_config_t* cfg, const void* q, int32_t q_frames,
+    const void* k_cache, const void* v_cache, int64_t cache_tokens,
+    int32_t num_segments, const int64_t* seg_start, const int64_t* seg_len,
+    void* out, float* lse, struct CUstream_st* stream);
+
 /* Number of kernel launches this plan has enqueued since it was created
  * (an append is one launch; an attention call is one, or two when the key
  * range of some query units is split across SMs and merged).  Host only. */

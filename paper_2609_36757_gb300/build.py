@@ -21,7 +21,8 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfastvr_attn.so")
 INCLUDE = os.path.join(ROOT, "include")
 
-SOURCES = ["fastvr_host.cpp", "kv_append.cu", "chunk_attn_fwd.cu"]
+SOURCES = ["fastvr_host.cpp", "kv_append.cu", "chunk_attn_fwd.cu",
+           "chunk_attn_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",
          "-Xcompiler", "-fvisibility=hidden", "-I", INCLUDE, "-I", CSRC]

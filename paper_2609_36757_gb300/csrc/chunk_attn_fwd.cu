@@ -78,7 +78,8 @@ struct TcParams {
   // fastest; the first units_full run whole, the rest are cut into `split`
   // key-tile ranges whose partial results go to the workspace.
   int32_t q_pairs, units_full, split;
-  float* ws;
+  float* ws;      // partial O: [part][d][kUnitRows]
+  float* ws_lse;  // partial log2-domain LSE: [part][kUnitRows]
 };
 
 // The work of one CTA.
@@ -449,8 +450,7 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     // Partial result of a key range: O / l in fp32 (transposed, so a warp's
     // stores are contiguous) and the log2-domain log-sum-exp.
     float* ws_o = p.ws + (size_t)w.part * D * kUnitRows;
-    float* ws_l = p.ws + (size_t)kMaxParts * D * kUnitRows +
-                  (size_t)w.part * kUnitRows;
+    float* ws_l = p.ws_lse + (size_t)w.part * kUnitRows;
 #pragma unroll
     for (int c = 0; c < D / 32; ++c) {
       uint32_t r[32];
@@ -504,7 +504,7 @@ combine_kernel(const __grid_constant__ TcParams p) {
   const int row = pair * kQTiles * kBM + r_unit;
   if (row >= p.q_tokens) return;
   const int k0 = ut * p.split;
-  const float* ws_l = p.ws + (size_t)kMaxParts * D * kUnitRows;
+  const float* ws_l = p.ws_lse;
   float m = -INFINITY;
   for (int i = 0; i < p.split; ++i)
     m = fmaxf(m, ws_l[(size_t)(k0 + i) * kUnitRows + r_unit]);
@@ -633,6 +633,32 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
+// Units of two query tiles: whole waves of units run whole, and the units of
+// a last partial wave are cut along the keys so that every SM has work (at
+// least kMinTilesPerPart key tiles per part, at most max_parts parts).
+void split_units(int units, int tiles, int sms, int max_parts, int* units_full,
+                 int* split) {
+  const int rem = units % sms;
+  int s = 1;
+  if (rem > 0) {
+    s = std::min(sms / rem, tiles / kMinTilesPerPart);
+    s = std::min(s, std::min(kMaxParts, max_parts) / rem);
+  }
+  if (s >= 2) {
+    *units_full = units - rem;
+    *split = s;
+  } else {
+    *units_full = units;
+    *split = 1;
+  }
+}
+
+int total_tiles(const AttnParams& a) {
+  int tiles = 0;
+  for (int s = 0; s < a.num_segments; ++s) tiles += (a.seg_len[s] + kBN - 1) / kBN;
+  return tiles;
+}
+
 bool make_map(CUtensorMap* m, const void* base, int d, int64_t tokens,
               int heads, int batch, int64_t token_stride_b,
               int64_t head_stride_b, int64_t batch_stride_b) {
@@ -687,25 +713,11 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
   p.inject_stall = a.inject_stall;
   p.ws = a.workspace;
 
-  // Units of two query tiles; whole waves of units run whole, and the units
-  // of a last partial wave are cut along the keys so that every SM has work
-  // (at least kMinTilesPerPart key tiles per part).
-  const int sms = sm_count();
   p.q_pairs = (a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);
   const int units = p.q_pairs * a.heads * a.batch;
-  const int rem = units % sms;
-  int split = 1;
-  if (rem > 0) {
-    split = std::min(sms / rem, tiles / kMinTilesPerPart);
-    split = std::min(split, kMaxParts / rem);
-  }
-  if (split >= 2) {
-    p.units_full = units - rem;
-    p.split = split;
-  } else {
-    p.units_full = units;
-    p.split = 1;
-  }
+  split_units(units, tiles, sm_count(), a.workspace_parts, &p.units_full,
+              &p.split);
+  p.ws_lse = p.ws + (size_t)a.workspace_parts * D * kUnitRows;
   const int grid = p.units_full + (units - p.units_full) * p.split;
   const int smem = Layout<D>::bytes;
   cudaError_t e = cudaFuncSetAttribute(
@@ -721,6 +733,14 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
 }
 
 }  // namespace
+
+int chunk_attn_parts(const AttnParams& a) {
+  const int pairs = (a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);
+  const int units = pairs * a.heads * a.batch;
+  int full = 0, split = 1;
+  split_units(units, total_tiles(a), sm_count(), kMaxParts, &full, &split);
+  return split > 1 ? (units - full) * split : 0;
+}
 
 cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream,
                               int* launches) {

@@ -264,6 +264,7 @@ fastvr_status_t fastvr_chunk_attn_fwd(fastvr_plan_t p, const void* q, void* out,
   a.scale_log2 = c.softmax_scale * 1.4426950408889634f;
   a.status = control_word(p);
   a.workspace = workspace(p);
+  a.workspace_parts = fastvr::kMaxParts;
   a.wait_limit_ns = p->wait_limit_ns;
   a.inject_stall = p->inject_stall;
   int launched = 0;

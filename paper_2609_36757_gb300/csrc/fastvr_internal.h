@@ -57,12 +57,17 @@ struct AttnParams {
   int32_t seg_len[kMaxSegments];
   float scale_log2;       // softmax_scale * log2(e)
   int* status;            // control word (device)
-  float* workspace;       // workspace_bytes(head_dim) of scratch (device)
+  float* workspace;       // split-KV scratch (device): workspace_parts
+                          // partial results of kUnitRows x (d + 1) floats
+  int32_t workspace_parts;
   uint64_t wait_limit_ns; // bound of every in-kernel wait (0 = default)
   int32_t inject_stall;   // test hook: stall the MMA issuer until timeout
 };
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream);
+// Workspace parts (partial results) a launch of p uses on the current device
+// (0 when no unit is split), with at most kMaxParts parts.
+int chunk_attn_parts(const AttnParams& p);
 // Enqueues the attention kernel (and the merge kernel when the key range of
 // some units is split); *launches receives the number of kernels enqueued.
 cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream,

@@ -57,6 +57,10 @@ SIGNATURES = {
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64)]),
     "fastvr_plan_launch_count": (_I32, [_VP, ctypes.POINTER(_I64)]),
+    "fastvr_chunk_attn_fwd_static": (_I32, [_CFGP, _VP, _I32, _VP, _VP, _I64,
+                                            _I32, ctypes.POINTER(_I64),
+                                            ctypes.POINTER(_I64), _VP, _VP,
+                                            _VP]),
     "fastvr_debug_inject_stall": (_I32, [_VP, _I32, ctypes.c_uint64]),
     "fastvr_plan_destroy": (None, [_VP]),
     "fastvr_status_string": (ctypes.c_char_p, [_I32]),
@@ -150,6 +154,20 @@ def fastvr_plan_visible(plan: int):
     _check(lib.fastvr_plan_visible(plan, ctypes.byref(n), st, ln,
                                    ctypes.byref(tot)), "fastvr_plan_visible")
     return [(st[i], ln[i]) for i in range(n.value)], tot.value
+
+
+def fastvr_chunk_attn_fwd_static(cfg: fastvr_attn_config_t, q: int,
+                                 q_frames: int, k_cache: int, v_cache: int,
+                                 cache_tokens: int, segments, out: int,
+                                 lse: int, stream: int) -> None:
+    """The allocation-free attention entry point; `segments` is a list of
+    (start, len) key ranges of one head's cache."""
+    n = len(segments)
+    st = (_I64 * max(2, n))(*[s for s, _ in segments])
+    ln = (_I64 * max(2, n))(*[l for _, l in segments])
+    _check(lib.fastvr_chunk_attn_fwd_static(
+        ctypes.byref(cfg), q, q_frames, k_cache, v_cache, cache_tokens, n, st,
+        ln, out, lse, stream), "fastvr_chunk_attn_fwd_static")
 
 
 def fastvr_plan_launch_count(plan: int) -> int:

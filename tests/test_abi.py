@@ -209,3 +209,28 @@ def test_visible_counts_match_oracle_pair_counts(fv):
             assert f * N * lk == want[c]
     finally:
         fv.fastvr_plan_destroy(plan)
+
+
+def test_static_entry_rejects_bad_arguments_before_any_device_work(fv):
+    cfg = fv.make_config(1, 2, 128, 64, 2, -1, 4)
+    ok_seg = [(0, 128)]
+    cases = [
+        dict(q=0), dict(q_frames=0), dict(cache_tokens=0),
+        dict(segments=[(0, 64)] * 3), dict(segments=[(0, 0)]),
+        dict(segments=[(200, 100)]), dict(segments=[(-1, 10)]),
+        dict(q=FAKE + 8), dict(out=FAKE + 4),
+    ]
+    for kw in cases:
+        a = dict(q=FAKE, q_frames=1, k=FAKE, v=FAKE, cache_tokens=256,
+                 segments=ok_seg, out=FAKE)
+        a.update(kw)
+        with pytest.raises(fv.FastVRError) as e:
+            fv.fastvr_chunk_attn_fwd_static(cfg, a["q"], a["q_frames"], a["k"],
+                                            a["v"], a["cache_tokens"],
+                                            a["segments"], a["out"], 0, 0)
+        assert e.value.status == fv.FASTVR_ERR_INVALID_ARG, kw
+    bad_d = fv.make_config(1, 2, 96, 64, 2, -1, 4)
+    with pytest.raises(fv.FastVRError) as e:
+        fv.fastvr_chunk_attn_fwd_static(bad_d, FAKE, 1, FAKE, FAKE, 256, ok_seg,
+                                        FAKE, 0, 0)
+    assert e.value.status == fv.FASTVR_ERR_UNSUPPORTED
