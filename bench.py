@@ -305,7 +305,12 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
     per_chunk_fwd = [statistics.median(fwd_ms[s][c] for s in range(args.steps))
                      for c in range(w.num_chunks)]
     peak = peaks["bf16_tflops_sustained"]
-    traffic = load_traffic("chunk_attn_fwd_1080p")
+    traffic = (load_traffic("chunk_attn_fwd_1080p") if w.name == "1080p"
+               else None)
+    kv_row = 2 * w.batch * w.heads * w.head_dim * 2  # K+V bytes per token
+    qkv_step = sum(3 * w.batch * w.heads * w.head_dim * 2 *
+                   w.frames_in_chunk(c) * w.tokens_per_frame
+                   for c in range(w.num_chunks))
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
@@ -316,9 +321,12 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
                    "head_dim": w.head_dim, "tokens_per_frame": w.tokens_per_frame,
                    "frames_per_chunk": w.frames_per_chunk,
                    "chunks": w.num_chunks, "window_chunks": w.window_chunks,
-                   "step": "reset + 15 x (kv_append + chunk_attn_fwd)",
-                   "l2": "inputs larger than L2 (visible K/V per chunk "
-                         "0.1-1.5 GB, 2.3 GB of Q/K/V per step)",
+                   "step": f"reset + {w.num_chunks} x (kv_append + "
+                           "chunk_attn_fwd)",
+                   "l2": f"inputs larger than L2 (visible K/V per chunk "
+                         f"{min(lk) * kv_row / 1e9:.2f}-"
+                         f"{max(lk) * kv_row / 1e9:.2f} GB, "
+                         f"{qkv_step / 1e9:.2f} GB of Q/K/V per step)",
                    "parallelism": f"replicas x{world} (one video per GPU)"},
         "ms_per_chunk": {"mean_fwd": statistics.mean(per_chunk_fwd),
                          "last_fwd": per_chunk_fwd[-1],
@@ -331,7 +339,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
         "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peak,
                      "unit": "TFLOP/s", "frac": attn_tflops / peak,
                      "peak_kind": f"{peak_kind} bf16 sustained",
-                     "kernel": "chunk_attn_fwd",
+                     "kernel": "chunk_attn_fwd (attention + split merge)",
                      "traffic": traffic},
         "gpu_launches": launches,
         "clocks": clock_info,
@@ -425,6 +433,7 @@ def reduce_max(x: float, world: int) -> float:
 
 
 def main(argv=None):
+    global WORKLOAD
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
@@ -432,6 +441,9 @@ def main(argv=None):
     ap.add_argument("--impl", default="fastvr", choices=["fastvr", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU-baseline sample length (0 skips it)")
+    ap.add_argument("--workload", default=WORKLOAD.name,
+                    choices=sorted(WL.WORKLOADS),
+                    help="workload to stream (the metric is quoted on 1080p)")
     ap.add_argument("--chunks", type=int, default=0,
                     help="stream only the first N chunks (small profiling "
                          "cases); 0 = the whole workload")
@@ -441,7 +453,7 @@ def main(argv=None):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    global WORKLOAD
+    WORKLOAD = WL.WORKLOADS[args.workload]
     if args.chunks:
         import dataclasses
         WORKLOAD = dataclasses.replace(WORKLOAD, num_chunks=args.chunks,

@@ -150,6 +150,24 @@ FASTVR_API fastvr_status_t fastvr_plan_visible(fastvr_plan_t plan, int32_t* num_
                                     int64_t* seg_start, int64_t* seg_len,
                                     int64_t* visible_tokens);
 
+/* One-shot chunk-causal attention over a whole sequence: the training form
+ * of Sec. 3.1, where the entire latent sequence is processed in parallel
+ * under the mask M of Eq. 1 (window cfg.window_chunks, -1 = every earlier
+ * chunk).  q, k, v: bfloat16 [B, L, H, d] token-major with L = num_frames *
+ * N; out bfloat16 [B, L, H, d]; lse nullable, float32 [B, H, L].  Frame f
+ * belongs to chunk f / k; a ragged final chunk is simply shorter.  Each
+ * block of 256 query rows reads only the keys its rows can see (invisible
+ * chunks are never loaded); rows that straddle a chunk boundary are masked
+ * element-wise.  No plan, no cache and no scratch memory are involved; a
+ * bounded-wait timeout leaves out undefined and is not reported.  The result
+ * equals the streamed form (fastvr_kv_append + fastvr_chunk_attn_fwd, chunk
+ * by chunk) up to rounding.
+ * Errors: INVALID_ARG, UNSUPPORTED (head_dim, device not sm_103), CUDA. */
+FASTVR_API fastvr_status_t fastvr_blockcausal_attn_fwd(
+    const fastvr_attn_config_t* cfg, int32_t num_frames, const void* q,
+    const void* k, const void* v, void* out, float* lse,
+    struct CUstream_st* stream);
+
 /* Chunk-causal attention that allocates nothing (no counterpart in the
  * paper; an interface for callers that cannot allocate device memory).
  * Callers such as serving runtimes that own all device memory through their

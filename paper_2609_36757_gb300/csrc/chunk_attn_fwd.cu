@@ -80,6 +80,9 @@ struct TcParams {
   int32_t q_pairs, units_full, split;
   float* ws;      // partial O: [part][d][kUnitRows]
   float* ws_lse;  // partial log2-domain LSE: [part][kUnitRows]
+  // One-shot (training-form) launches: the whole sequence of seq_tokens
+  // tokens, chunks of chunk_tokens tokens, window W (-1: unbounded).
+  int32_t seq_tokens, chunk_tokens, window, batch;
 };
 
 // The work of one CTA.
@@ -88,10 +91,37 @@ struct Work {
   int j0, n;   // first key tile (index into the visible tiles) and count
   int nqt;     // query tiles with at least one row in the chunk (1 or 2)
   int part;    // -1: whole unit, final output; else workspace slot
+  int kv0, kv1;  // one-shot: the unit's key token range [kv0, kv1)
 };
 
-__device__ __forceinline__ Work cta_work(const TcParams& p) {
+// One-shot launches: unit x covers query pair nq - 1 - x / (H B) of head
+// x % H, batch (x / H) % B, so the units with the most keys start first.
+// Its keys are the union of what its rows see: chunks max(0, c_lo - W) ..
+// c_hi of the unit's first and last rows (Eq. 1 with window W).
+__device__ __forceinline__ Work oneshot_work(const TcParams& p) {
   Work w;
+  const int bh = blockIdx.x % (p.heads * p.batch);
+  const int pair = p.q_pairs - 1 - blockIdx.x / (p.heads * p.batch);
+  w.h = bh % p.heads;
+  w.b = bh / p.heads;
+  w.q0 = pair * kQTiles * kBM;
+  w.nqt = (p.q_tokens - w.q0 > kBM) ? 2 : 1;
+  const int c_lo = w.q0 / p.chunk_tokens;
+  const int c_hi = min(w.q0 + kQTiles * kBM, p.q_tokens) - 1;
+  const int chunk_hi = c_hi / p.chunk_tokens;
+  w.kv0 = p.window < 0 ? 0 : max(0, c_lo - p.window) * p.chunk_tokens;
+  w.kv1 = min((chunk_hi + 1) * p.chunk_tokens, p.seq_tokens);
+  w.j0 = 0;
+  w.n = (w.kv1 - w.kv0 + kBN - 1) / kBN;
+  w.part = -1;
+  return w;
+}
+
+template <bool kOneShot>
+__device__ __forceinline__ Work cta_work(const TcParams& p) {
+  if (kOneShot) return oneshot_work(p);
+  Work w;
+  w.kv0 = w.kv1 = 0;
   int unit, part = -1, nparts = 1, idx = 0;
   if ((int)blockIdx.x < p.units_full) {
     unit = blockIdx.x;
@@ -160,7 +190,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
     if (*reinterpret_cast<volatile int*>(&S->abort)) return false;
     if (global_timer_ns() - t0 > S->wait_limit_ns) {
       *reinterpret_cast<volatile int*>(&S->abort) = 1;
-      atomicExch(status, kDevTimeout);
+      if (status != nullptr) atomicExch(status, kDevTimeout);
       return false;
     }
   }
@@ -175,6 +205,14 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity,
   }
 }
 
+// One-shot: key tile j of the unit range [kv0, kv1) (map 0).
+__device__ __forceinline__ void oneshot_tile(int kv0, int kv1, int j,
+                                             int& seg, int& tok0, int& valid) {
+  seg = 0;
+  tok0 = kv0 + j * kBN;
+  valid = min(kBN, kv1 - tok0);
+}
+
 __device__ __forceinline__ void tile_coord(const TcParams& p, int j, int& seg,
                                            int& tok0, int& valid) {
   seg = j < p.seg_tiles0 ? 0 : 1;
@@ -186,7 +224,7 @@ __device__ __forceinline__ void tile_coord(const TcParams& p, int j, int& seg,
 // TMA producers, one thread each: the K producer also loads the query tiles.
 // K and V advance independently, so a slow V slot never holds back the next
 // K tile (QK^T of tile j+1 is issued before PV of tile j completes).
-template <int D, bool kIsK>
+template <int D, bool kIsK, bool kOneShot>
 __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
                          const Work& w) {
   const int h = w.h, b = w.b;
@@ -209,7 +247,10 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
     const int st = j % kStages;
     const uint32_t ph = (j / kStages) & 1;
     int seg, tok0, valid;
-    tile_coord(p, w.j0 + j, seg, tok0, valid);
+    if (kOneShot)
+      oneshot_tile(w.kv0, w.kv1, j, seg, tok0, valid);
+    else
+      tile_coord(p, w.j0 + j, seg, tok0, valid);
     if (!wait_bar(&empty[st], ph ^ 1, S, p.status)) break;
     mbar_arrive_expect_tx(&full[st], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
@@ -378,9 +419,29 @@ __device__ __forceinline__ void mask_max32(uint32_t (&sc)[32], int c, int valid,
                      __uint_as_float(sc[2 * i + 1]));
 }
 
-template <int D>
+// One-shot: mask the columns of s[c] outside this row's visible range
+// [lo, hi) (relative to the tile) and fold the row max as mask_max32 does.
+__device__ __forceinline__ void mask_range_max32(uint32_t (&sc)[32], int c,
+                                                 int lo, int hi,
+                                                 float (&mx)[4]) {
+  if (lo > c * 32 || hi < (c + 1) * 32) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (c * 32 + i < lo || c * 32 + i >= hi) sc[i] = 0xff800000u;  // -inf
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    mx[i & 3] = max3(mx[i & 3], __uint_as_float(sc[2 * i]),
+                     __uint_as_float(sc[2 * i + 1]));
+}
+
+// Streaming: j0, n index the launch's visible tiles.  One-shot: the tiles of
+// [kv0, kv1); a row of chunk c sees keys of chunks max(0, c - W) .. c, so a
+// row can be fully masked in a tile (its reference then stays at -inf).
+template <int D, bool kOneShot>
 __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
-                             int t, int wq, int lane, int j0, int n) {
+                             int t, int wq, int lane, int j0, int n, int kv0,
+                             int kv1, int q0) {
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
   const uint32_t tS = tmem + t * 128 + lane_off;
   const uint32_t tO = tmem + 256 + t * 128 + lane_off;
@@ -389,9 +450,19 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   float m_ref = -INFINITY;  // exp2-domain reference (scaled scores)
   float l = 0.f;
   bool ok = true;
+  int vis_lo = 0, vis_hi = 0;  // one-shot: this row's visible key tokens
+  if (kOneShot) {
+    const int row = min(q0 + t * kBM + wq * 32 + lane, p.q_tokens - 1);
+    const int c = row / p.chunk_tokens;
+    vis_lo = p.window < 0 ? 0 : max(0, c - p.window) * p.chunk_tokens;
+    vis_hi = min((c + 1) * p.chunk_tokens, p.seq_tokens);
+  }
   for (int j = 0; j < n; ++j) {
     int seg, tok0, valid;
-    tile_coord(p, j0 + j, seg, tok0, valid);
+    if (kOneShot)
+      oneshot_tile(kv0, kv1, j, seg, tok0, valid);
+    else
+      tile_coord(p, j0 + j, seg, tok0, valid);
     if (!(ok = wait_bar(&S->s_full[t], j & 1, S, p.status))) break;
     tc_fence_after();
     uint32_t s[4][32];
@@ -401,11 +472,21 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     tmem_ld32(tS + 64, s[2]);  // lands while the first half is reduced
     tmem_ld32(tS + 96, s[3]);
     float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-    mask_max32(s[0], 0, valid, mx);
-    mask_max32(s[1], 1, valid, mx);
-    tmem_wait_ld();
-    mask_max32(s[2], 2, valid, mx);
-    mask_max32(s[3], 3, valid, mx);
+    if (kOneShot) {
+      const int lo = vis_lo - tok0;
+      const int hi = min(vis_hi - tok0, valid);
+      mask_range_max32(s[0], 0, lo, hi, mx);
+      mask_range_max32(s[1], 1, lo, hi, mx);
+      tmem_wait_ld();
+      mask_range_max32(s[2], 2, lo, hi, mx);
+      mask_range_max32(s[3], 3, lo, hi, mx);
+    } else {
+      mask_max32(s[0], 0, valid, mx);
+      mask_max32(s[1], 1, valid, mx);
+      tmem_wait_ld();
+      mask_max32(s[2], 2, valid, mx);
+      mask_max32(s[3], 3, valid, mx);
+    }
     const float mrow = fmaxf(max3(mx[0], mx[1], mx[2]), mx[3]) * sl2;
     // The reference moves only when a row max passes it by more than the
     // threshold (decided per warp: TMEM accesses are warp-wide).
@@ -415,10 +496,13 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     if (rescale) {
       const float m_new = fmaxf(m_ref, mrow);
       alpha = ex2(m_ref - m_new);
+      if (kOneShot && m_new == -INFINITY) alpha = 1.f;  // still nothing seen
       l *= alpha;
       m_ref = m_new;
     }
-    const uint64_t neg2 = f2_pack(-m_ref, -m_ref);
+    // A row that has seen no visible key yet exponentiates -inf against 0.
+    const float neg = (kOneShot && m_ref == -INFINITY) ? 0.f : -m_ref;
+    const uint64_t neg2 = f2_pack(neg, neg);
     uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
     for (int c = 0; c < 4; ++c) exp_store32(s[c], sl2x2, neg2, tS + 16 * c, acc);
@@ -442,7 +526,7 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   }
   if (!ok || !wait_bar(&S->o_full, 0, S, p.status)) return;
   tc_fence_after();
-  const Work w = cta_work(p);
+  const Work w = cta_work<kOneShot>(p);
   const int r_unit = t * kBM + wq * 32 + lane;  // row within the unit
   const int row = w.q0 + r_unit;
   const float inv_l = 1.f / l;
@@ -491,56 +575,68 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
 
 // Merge the partial results of the split units: weights 2^(lse_i - m),
 // O = sum_i w_i O_i / sum_i w_i, LSE = m + log2(sum_i w_i) (natural log out).
-// One thread per query row, 128 rows per CTA; workspace reads are coalesced.
+// A CTA merges 32 query rows of one unit: thread (r, g) accumulates columns
+// [16 g, 16 g + 16) of row r, so a warp reads 32 consecutive rows of one
+// column of a part (coalesced); the bf16 rows are then written contiguously
+// through shared memory.
+constexpr int kMergeRows = 32;
+
 template <int D>
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(kMergeRows * D / 16)
 combine_kernel(const __grid_constant__ TcParams p) {
+  constexpr int kCols = 16;  // columns per thread
+  __shared__ __align__(16) uint16_t tile[kMergeRows][D + 8];
   const int ut = blockIdx.x;
-  const int r_unit = blockIdx.y * 128 + threadIdx.x;
+  const int r = threadIdx.x % kMergeRows;
+  const int g = threadIdx.x / kMergeRows;
+  const int r_unit = blockIdx.y * kMergeRows + r;
   const int unit = p.units_full + ut;
   const int pair = unit % p.q_pairs;
   const int h = (unit / p.q_pairs) % p.heads;
   const int b = unit / (p.q_pairs * p.heads);
-  const int row = pair * kQTiles * kBM + r_unit;
-  if (row >= p.q_tokens) return;
+  const int row0 = pair * kQTiles * kBM + blockIdx.y * kMergeRows;
+  if (row0 >= p.q_tokens) return;  // the whole block is past the chunk end
   const int k0 = ut * p.split;
-  const float* ws_l = p.ws_lse;
   float m = -INFINITY;
   for (int i = 0; i < p.split; ++i)
-    m = fmaxf(m, ws_l[(size_t)(k0 + i) * kUnitRows + r_unit]);
+    m = fmaxf(m, p.ws_lse[(size_t)(k0 + i) * kUnitRows + r_unit]);
+  float acc[kCols];
+#pragma unroll
+  for (int x = 0; x < kCols; ++x) acc[x] = 0.f;
   float wsum = 0.f;
-  for (int i = 0; i < p.split; ++i)
-    wsum += ex2(ws_l[(size_t)(k0 + i) * kUnitRows + r_unit] - m);
-  const float inv = 1.f / wsum;
-  uint16_t* orow = p.o + (int64_t)b * p.o_str.batch +
-                   (int64_t)row * p.o_str.token + (int64_t)h * p.o_str.head;
-#pragma unroll 1
-  for (int c = 0; c < D / 32; ++c) {
-    float acc[32];
+  for (int i = 0; i < p.split; ++i) {
+    const float wi = ex2(p.ws_lse[(size_t)(k0 + i) * kUnitRows + r_unit] - m);
+    wsum += wi;
+    const float* src =
+        p.ws + ((size_t)(k0 + i) * D + g * kCols) * kUnitRows + r_unit;
+    float v[kCols];
 #pragma unroll
-    for (int x = 0; x < 32; ++x) acc[x] = 0.f;
-    for (int i = 0; i < p.split; ++i) {
-      const float wi =
-          ex2(ws_l[(size_t)(k0 + i) * kUnitRows + r_unit] - m) * inv;
-      const float* src =
-          p.ws + ((size_t)(k0 + i) * D + c * 32) * kUnitRows + r_unit;
+    for (int x = 0; x < kCols; ++x) v[x] = src[x * kUnitRows];
 #pragma unroll
-      for (int x = 0; x < 32; ++x) acc[x] = fmaf(wi, src[x * kUnitRows], acc[x]);
-    }
-    uint32_t pk[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) pk[i] = pack_bf16(acc[2 * i], acc[2 * i + 1]);
-    uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
-#pragma unroll
-    for (int v = 0; v < 4; ++v)
-      dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+    for (int x = 0; x < kCols; ++x) acc[x] = fmaf(wi, v[x], acc[x]);
   }
-  if (p.lse != nullptr)
-    p.lse[((int64_t)b * p.heads + h) * p.q_tokens + row] =
+  const float inv = 1.f / wsum;
+#pragma unroll
+  for (int x = 0; x < kCols; x += 2)
+    *reinterpret_cast<uint32_t*>(&tile[r][g * kCols + x]) =
+        pack_bf16(acc[x] * inv, acc[x + 1] * inv);
+  if (g == 0 && p.lse != nullptr && row0 + r < p.q_tokens)
+    p.lse[((int64_t)b * p.heads + h) * p.q_tokens + row0 + r] =
         (m + __log2f(wsum)) * 0.6931471805599453f;
+  __syncthreads();
+  // Each row is d bf16 = D / 8 16-byte pieces; one piece per thread.
+  for (int i = threadIdx.x; i < kMergeRows * D / 8; i += blockDim.x) {
+    const int rr = i / (D / 8), piece = i % (D / 8);
+    const int row = row0 + rr;
+    if (row < p.q_tokens)
+      *reinterpret_cast<uint4*>(p.o + (int64_t)b * p.o_str.batch +
+                                (int64_t)row * p.o_str.token +
+                                (int64_t)h * p.o_str.head + piece * 8) =
+          *reinterpret_cast<const uint4*>(&tile[rr][piece * 8]);
+  }
 }
 
-template <int D>
+template <int D, bool kOneShot>
 __global__ void __launch_bounds__(kThreads, 1)
 chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   using L = Layout<D>;
@@ -550,7 +646,7 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   Shared* S = reinterpret_cast<Shared*>(smem + L::shared_off);
   const int warp = threadIdx.x / 32;
   const int lane = threadIdx.x % 32;
-  const Work w = cta_work(p);
+  const Work w = cta_work<kOneShot>(p);
 
   if (warp == 9) {
     tmem_alloc(&S->tmem_base, kTmemCols);
@@ -582,10 +678,10 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   const uint32_t tmem = S->tmem_base;
 
   if (warp == 8) {
-    if (lane == 0) producer<D, true>(p, smem, S, w);
+    if (lane == 0) producer<D, true, kOneShot>(p, smem, S, w);
     __syncwarp();
   } else if (warp == 10) {
-    if (lane == 0) producer<D, false>(p, smem, S, w);
+    if (lane == 0) producer<D, false, kOneShot>(p, smem, S, w);
     __syncwarp();
   } else if (warp == 9) {
     if (lane == 0) mma_issuer<D>(p, smem, S, tmem, w);
@@ -593,7 +689,8 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   } else {
     // A query tile that lies past the end of the chunk has no work.
     if (warp / 4 < w.nqt)
-      softmax_role<D>(p, S, tmem, warp / 4, warp % 4, lane, w.j0, w.n);
+      softmax_role<D, kOneShot>(p, S, tmem, warp / 4, warp % 4, lane, w.j0,
+                                w.n, w.kv0, w.kv1, w.q0);
   }
   tc_fence_before();
   __syncthreads();
@@ -721,18 +818,69 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
   const int grid = p.units_full + (units - p.units_full) * p.split;
   const int smem = Layout<D>::bytes;
   cudaError_t e = cudaFuncSetAttribute(
-      chunk_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      chunk_attn_tc_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      smem);
   if (e != cudaSuccess) return e;
-  chunk_attn_tc_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+  chunk_attn_tc_kernel<D, false><<<grid, kThreads, smem, stream>>>(p);
   *launches = 1;
   if (p.split > 1) {
-    combine_kernel<D><<<dim3(units - p.units_full, kQTiles), 128, 0, stream>>>(p);
+    combine_kernel<D><<<dim3(units - p.units_full, kUnitRows / kMergeRows),
+                        kMergeRows * D / 16, 0, stream>>>(p);
     *launches = 2;
   }
   return cudaGetLastError();
 }
 
+// One unit per pair of query tiles, no key splitting: the units differ in
+// length (later chunks see more keys) and run longest first.
+template <int D>
+cudaError_t launch_oneshot_d(const OneShotParams& a, cudaStream_t stream) {
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  const int64_t es = 2;
+  const int64_t tok = (int64_t)a.heads * D, bat = (int64_t)a.seq_tokens * tok;
+  if (!make_map(&p.q_map, a.q, D, a.seq_tokens, a.heads, a.batch, tok * es,
+                D * es, bat * es) ||
+      !make_map(&p.k_map[0], a.k, D, a.seq_tokens, a.heads, a.batch, tok * es,
+                D * es, bat * es) ||
+      !make_map(&p.v_map[0], a.v, D, a.seq_tokens, a.heads, a.batch, tok * es,
+                D * es, bat * es))
+    return cudaErrorInvalidValue;
+  p.k_map[1] = p.k_map[0];
+  p.v_map[1] = p.v_map[0];
+  p.o = a.o;
+  p.lse = a.lse;
+  p.o_str.token = tok;
+  p.o_str.head = D;
+  p.o_str.batch = bat;
+  p.q_tokens = a.seq_tokens;
+  p.heads = a.heads;
+  p.batch = a.batch;
+  p.scale_log2 = a.scale_log2;
+  p.status = a.status;
+  p.seq_tokens = a.seq_tokens;
+  p.chunk_tokens = a.chunk_tokens;
+  p.window = a.window;
+  p.q_pairs = (a.seq_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);
+  p.split = 1;
+  const int grid = p.q_pairs * a.heads * a.batch;
+  p.units_full = grid;
+  const int smem = Layout<D>::bytes;
+  cudaError_t e = cudaFuncSetAttribute(
+      chunk_attn_tc_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      smem);
+  if (e != cudaSuccess) return e;
+  chunk_attn_tc_kernel<D, true><<<grid, kThreads, smem, stream>>>(p);
+  return cudaGetLastError();
+}
+
 }  // namespace
+
+cudaError_t launch_blockcausal_attn(const OneShotParams& p, cudaStream_t stream) {
+  if (p.head_dim == 64) return launch_oneshot_d<64>(p, stream);
+  if (p.head_dim == 128) return launch_oneshot_d<128>(p, stream);
+  return cudaErrorInvalidValue;
+}
 
 int chunk_attn_parts(const AttnParams& a) {
   const int pairs = (a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);

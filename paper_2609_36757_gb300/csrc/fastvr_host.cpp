@@ -340,6 +340,55 @@ fastvr_status_t fastvr_plan_visible(fastvr_plan_t p, int32_t* num_segments,
   return FASTVR_OK;
 }
 
+fastvr_status_t fastvr_blockcausal_attn_fwd(const fastvr_attn_config_t* cfg,
+                                            int32_t num_frames, const void* q,
+                                            const void* k, const void* v,
+                                            void* out, float* lse,
+                                            struct CUstream_st* stream) {
+  if (cfg == nullptr || cfg->batch < 1 || cfg->heads < 1 ||
+      cfg->tokens_per_frame < 1 || cfg->frames_per_chunk < 1 ||
+      cfg->window_chunks < -1 || !(cfg->softmax_scale >= 0.f) ||
+      !isfinite(cfg->softmax_scale) || num_frames < 1 || q == nullptr ||
+      k == nullptr || v == nullptr || out == nullptr || !aligned16(q) ||
+      !aligned16(k) || !aligned16(v) || !aligned16(out) ||
+      (((uintptr_t)lse) & 3u) != 0)
+    return FASTVR_ERR_INVALID_ARG;
+  if (!supported_dim(cfg->head_dim)) return FASTVR_ERR_UNSUPPORTED;
+  const int64_t L = (int64_t)num_frames * cfg->tokens_per_frame;
+  const int64_t chunk = (int64_t)cfg->frames_per_chunk * cfg->tokens_per_frame;
+  if (L > INT32_MAX / 2 || chunk > INT32_MAX / 2) return FASTVR_ERR_INVALID_ARG;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) !=
+          cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  if (major != 10 || minor != 3) return FASTVR_ERR_UNSUPPORTED;
+  fastvr::OneShotParams a;
+  memset(&a, 0, sizeof(a));
+  a.q = static_cast<const uint16_t*>(q);
+  a.k = static_cast<const uint16_t*>(k);
+  a.v = static_cast<const uint16_t*>(v);
+  a.o = static_cast<uint16_t*>(out);
+  a.lse = lse;
+  a.batch = cfg->batch;
+  a.heads = cfg->heads;
+  a.head_dim = cfg->head_dim;
+  a.seq_tokens = (int32_t)L;
+  a.chunk_tokens = (int32_t)chunk;
+  a.window = cfg->window_chunks;
+  const float scale = cfg->softmax_scale == 0.f
+                          ? 1.f / sqrtf((float)cfg->head_dim)
+                          : cfg->softmax_scale;
+  a.scale_log2 = scale * 1.4426950408889634f;
+  a.status = nullptr;
+  if (fastvr::launch_blockcausal_attn(a, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  return FASTVR_OK;
+}
+
 fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t p, int64_t* launches) {
   if (p == nullptr || launches == nullptr) return FASTVR_ERR_INVALID_ARG;
   *launches = p->launches;

@@ -65,6 +65,22 @@ struct AttnParams {
 };
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream);
+// One-shot (training-form) attention over a whole token-major sequence.
+struct OneShotParams {
+  const uint16_t* q;      // bfloat16 [B, L, H, d] token-major
+  const uint16_t* k;
+  const uint16_t* v;
+  uint16_t* o;            // bfloat16 [B, L, H, d]
+  float* lse;             // float32 [B, H, L] or null
+  int32_t batch, heads, head_dim;
+  int32_t seq_tokens;     // L = frames * tokens per frame
+  int32_t chunk_tokens;   // k * N
+  int32_t window;         // W, -1 = unbounded
+  float scale_log2;
+  int* status;            // control word or null (timeouts not reported)
+};
+cudaError_t launch_blockcausal_attn(const OneShotParams& p, cudaStream_t stream);
+
 // Workspace parts (partial results) a launch of p uses on the current device
 // (0 when no unit is split), with at most kMaxParts parts.
 int chunk_attn_parts(const AttnParams& p);

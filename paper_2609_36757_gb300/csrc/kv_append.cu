@@ -8,53 +8,71 @@
 // vector accesses.  Consecutive threads read consecutive 16-byte pieces of the
 // source, and the d/8 pieces of one (token, head) row land contiguously in the
 // cache, so both sides are fully coalesced at 32-byte sector granularity.
+// Each thread keeps eight loads in flight before it stores (enough bytes in
+// flight to cover HBM latency with a few CTAs per SM); the source is read
+// with an evict-first hint since it is not read again.
 #include "fastvr_internal.h"
 
 namespace fastvr {
 namespace {
 
-__global__ void __launch_bounds__(256)
-kv_append_kernel(AppendParams p) {
-  const int vec_per_row = p.head_dim / 8;  // 16-byte vectors per (t, h) row
-  const int64_t per_tensor =
-      (int64_t)p.batch * p.tokens * p.heads * vec_per_row;
-  const int64_t total = 2 * per_tensor;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-       i += stride) {
-    const bool is_v = i >= per_tensor;
-    const int64_t j = is_v ? i - per_tensor : i;
-    const int vec = (int)(j % vec_per_row);
-    int64_t r = j / vec_per_row;
-    const int h = (int)(r % p.heads);
-    r /= p.heads;
-    const int64_t t = r % p.tokens;
-    const int64_t b = r / p.tokens;
-    const uint4* src = reinterpret_cast<const uint4*>(is_v ? p.v_new : p.k_new);
-    uint4* dst = reinterpret_cast<uint4*>(is_v ? p.v_cache : p.k_cache);
-    const int64_t d_idx =
-        ((b * p.heads + h) * p.cache_tokens + p.token_offset + t) * vec_per_row +
-        vec;
-    dst[d_idx] = __ldg(src + j);
+constexpr int kUnroll = 8;
+
+template <int VPR>  // 16-byte vectors per (token, head) row: d / 8
+__device__ __forceinline__ int64_t cache_index(const AppendParams& p,
+                                               uint32_t j) {
+  const uint32_t vec = j % VPR;
+  const uint32_t r = j / VPR;  // (b, t, h) row, h fastest
+  const uint32_t h = r % (uint32_t)p.heads;
+  const uint32_t bt = r / (uint32_t)p.heads;
+  const uint32_t t = bt % (uint32_t)p.tokens;
+  const uint32_t b = bt / (uint32_t)p.tokens;
+  return (((int64_t)b * p.heads + h) * p.cache_tokens + p.token_offset + t) *
+             VPR + vec;
+}
+
+// blockIdx.y selects K (0) or V (1).
+template <int VPR>
+__global__ void __launch_bounds__(256) kv_append_kernel(AppendParams p) {
+  const uint4* src =
+      reinterpret_cast<const uint4*>(blockIdx.y ? p.v_new : p.k_new);
+  uint4* dst = reinterpret_cast<uint4*>(blockIdx.y ? p.v_cache : p.k_cache);
+  const uint32_t n = (uint32_t)p.batch * p.tokens * p.heads * VPR;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+  for (; i + (kUnroll - 1) * stride < n; i += kUnroll * stride) {
+    uint4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) v[u] = __ldcs(src + i + u * stride);
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+      dst[cache_index<VPR>(p, i + u * stride)] = v[u];
   }
+  for (; i < n; i += stride) dst[cache_index<VPR>(p, i)] = __ldcs(src + i);
 }
 
 }  // namespace
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream) {
-  const int64_t total =
-      2LL * p.batch * p.tokens * p.heads * (p.head_dim / 8);
-  if (total == 0) return cudaSuccess;
+  const int vpr = p.head_dim / 8;
+  const int64_t n = (int64_t)p.batch * p.tokens * p.heads * vpr;
+  if (n == 0) return cudaSuccess;
+  if (n > 0x7fffffffLL) return cudaErrorInvalidValue;  // 32-bit indexing
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (sms <= 0) sms = 152;
-  // Enough resident threads to cover HBM latency: 8 CTAs of 256 per SM,
-  // never more CTAs than work.
-  int64_t blocks = (int64_t)sms * 8;
-  const int64_t need = (total + 255) / 256;
+  // Four CTAs of 256 threads per SM and tensor, never more than the work.
+  int64_t blocks = (int64_t)sms * 4;
+  const int64_t need = (n + 255) / 256;
   if (blocks > need) blocks = need;
-  kv_append_kernel<<<(unsigned)blocks, 256, 0, stream>>>(p);
+  const dim3 grid((unsigned)blocks, 2);
+  if (vpr == 16)
+    kv_append_kernel<16><<<grid, 256, 0, stream>>>(p);
+  else if (vpr == 8)
+    kv_append_kernel<8><<<grid, 256, 0, stream>>>(p);
+  else
+    return cudaErrorInvalidValue;
   return cudaGetLastError();
 }
 

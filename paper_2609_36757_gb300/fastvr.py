@@ -57,6 +57,8 @@ SIGNATURES = {
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64)]),
     "fastvr_plan_launch_count": (_I32, [_VP, ctypes.POINTER(_I64)]),
+    "fastvr_blockcausal_attn_fwd": (_I32, [_CFGP, _I32, _VP, _VP, _VP, _VP,
+                                           _VP, _VP]),
     "fastvr_chunk_attn_fwd_static": (_I32, [_CFGP, _VP, _I32, _VP, _VP, _I64,
                                             _I32, ctypes.POINTER(_I64),
                                             ctypes.POINTER(_I64), _VP, _VP,
@@ -168,6 +170,38 @@ def fastvr_chunk_attn_fwd_static(cfg: fastvr_attn_config_t, q: int,
     _check(lib.fastvr_chunk_attn_fwd_static(
         ctypes.byref(cfg), q, q_frames, k_cache, v_cache, cache_tokens, n, st,
         ln, out, lse, stream), "fastvr_chunk_attn_fwd_static")
+
+
+def fastvr_blockcausal_attn_fwd(cfg: fastvr_attn_config_t, num_frames: int,
+                                q: int, k: int, v: int, out: int, lse: int,
+                                stream: int) -> None:
+    _check(lib.fastvr_blockcausal_attn_fwd(ctypes.byref(cfg), num_frames, q,
+                                           k, v, out, lse, stream),
+           "fastvr_blockcausal_attn_fwd")
+
+
+def blockcausal_attention(cfg: fastvr_attn_config_t, q, k, v,
+                          want_lse: bool = False):
+    """Torch convenience for fastvr_blockcausal_attn_fwd: q, k, v contiguous
+    bfloat16 CUDA tensors [B, L, H, d]; runs on the current stream."""
+    import torch
+    for t in (q, k, v):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError("q, k, v must be contiguous bfloat16 CUDA tensors")
+    if not (q.shape == k.shape == v.shape):
+        raise ValueError("q, k, v differ in shape")
+    B, L, H, d = q.shape
+    if (B, H, d) != (cfg.batch, cfg.heads, cfg.head_dim) or \
+            L % cfg.tokens_per_frame:
+        raise ValueError(f"q has shape {tuple(q.shape)}")
+    out = torch.empty_like(q)
+    lse = (torch.empty((B, H, L), dtype=torch.float32, device=q.device)
+           if want_lse else None)
+    fastvr_blockcausal_attn_fwd(cfg, L // cfg.tokens_per_frame, q.data_ptr(),
+                                k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                0 if lse is None else lse.data_ptr(),
+                                torch.cuda.current_stream().cuda_stream)
+    return (out, lse) if want_lse else out
 
 
 def fastvr_plan_launch_count(plan: int) -> int:

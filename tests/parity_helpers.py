@@ -55,7 +55,13 @@ class Err:
     def rel_l2(self) -> float:
         return (self.sq_err / max(self.sq_ref, 1e-300)) ** 0.5
 
+    def __str__(self) -> str:
+        return (f"max-abs {self.max_abs:.3e} mean-abs {self.mean_abs:.3e} "
+                f"rel-L2 {self.rel_l2:.3e} lse {self.lse_max:.3e} "
+                f"({self.count} elements)")
+
     def check(self) -> None:
+        print(f"parity: {self}")
         assert np.isfinite(self.max_abs), self
         assert self.max_abs <= MAX_ABS, self
         assert self.mean_abs <= MEAN_ABS, self
