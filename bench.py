@@ -292,6 +292,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
 
     e2e = (None if args.skip_e2e else
            run_e2e(args, w, chunks, att, dev, step_flops, world))
+    one_step = measure_one_step(dev)
 
     if rank != 0:
         return
@@ -342,6 +343,8 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
                      "kernel": "chunk_attn_fwd (attention + split merge)",
                      "traffic": traffic},
         "gpu_launches": launches,
+        "one_step_update": dict(one_step,
+                                frac_of_hbm=one_step["gbs"] / peaks["hbm_gbs"]),
         "clocks": clock_info,
         "e2e": e2e,
     }
@@ -351,6 +354,33 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
                                 "cores": HOST_CORES, "kind": "oracle",
                                 "sample": desc}
     print(json.dumps(line), flush=True)
+
+
+def measure_one_step(dev, sets: int = 8, rounds: int = 3):
+    """The one-step update z_hat = z_LQ - sigma v (Eq. one_step, outside the
+    attention step) on 1080p-sized latents: 48 channels x 30 latent frames x
+    68 x 120, bf16.  Successive calls rotate over `sets` distinct latents
+    (8 x 70 MB, larger than L2), timed with CUDA events; bytes = read z and
+    v, write z_hat."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    n = 48 * 30 * 68 * 120
+    bufs = [(torch.randn(n, device=dev).to(torch.bfloat16),
+             torch.randn(n, device=dev).to(torch.bfloat16),
+             torch.empty(n, device=dev, dtype=torch.bfloat16))
+            for _ in range(sets)]
+    for z, v, out in bufs:
+        FV.one_step_update(z, v, 0.8, out=out)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record()
+    for _ in range(rounds):
+        for z, v, out in bufs:
+            FV.one_step_update(z, v, 0.8, out=out)
+    end.record()
+    torch.cuda.synchronize(dev)
+    us = start.elapsed_time(end) * 1e3 / (rounds * sets)
+    return {"elements": n, "us": us, "gbs": 3 * 2 * n / (us * 1e-6) / 1e9,
+            "l2": f"{sets} distinct latents rotated ({sets * 6 * n / 1e6:.0f} MB)"}
 
 
 def run_e2e(args, w, chunks, att, dev, step_flops, world):

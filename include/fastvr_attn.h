@@ -168,6 +168,22 @@ FASTVR_API fastvr_status_t fastvr_blockcausal_attn_fwd(
     const void* k, const void* v, void* out, float* lse,
     struct CUstream_st* stream);
 
+/* FastVR's one-step restoration update (Eq. `eq:one_step`, used at
+ * inference and in Stage II training): z_hat = z_lq - sigma * v, with v the
+ * DiT's predicted velocity at t = tau and sigma = sigma_tau (an input: the
+ * shifted schedule's constants are not given in the paper).  Elementwise
+ * over n elements in any layout (the same for all three buffers); z_lq and
+ * z_hat are bfloat16 (dtype 0) or float32 (dtype 1), v is bfloat16.
+ * Computed as one fp32 FMA per element and rounded once (round to nearest
+ * even) to the output type.  z_hat may be z_lq (in place).  Pointers must be
+ * 16-byte aligned device addresses.
+ * Errors: INVALID_ARG, UNSUPPORTED (device not sm_103), CUDA. */
+FASTVR_API fastvr_status_t fastvr_one_step_update(const void* z_lq,
+                                                  const void* v, void* z_hat,
+                                                  int64_t n, float sigma,
+                                                  int32_t dtype,
+                                                  struct CUstream_st* stream);
+
 /* Chunk-causal attention that allocates nothing (no counterpart in the
  * paper; an interface for callers that cannot allocate device memory).
  * Callers such as serving runtimes that own all device memory through their

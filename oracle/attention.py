@@ -265,3 +265,38 @@ def visible_pairs_per_chunk(frames: Sequence[int], tokens_per_frame: int,
         lk = sum(frames[j] for j in visible_chunks(c, window))
         out.append(f * tokens_per_frame * lk * tokens_per_frame)
     return out
+
+
+# --------------------------------------------------------------------------
+# Backward of the one-shot form (gradients for training under the mask)
+# --------------------------------------------------------------------------
+def blockcausal_attention_bwd(q: np.ndarray, k: np.ndarray, v: np.ndarray,
+                              do: np.ndarray, tokens_per_frame: int,
+                              frames_per_chunk: int, window: int,
+                              scale: float):
+    """Gradients of the one-shot chunk-causal attention (training form,
+    Sec. 3.1: the whole sequence under M) with respect to q, k and v, given
+    the output gradient do; all [B, L, H, d] float64.
+
+    With s_ij = scale <q_i, k_j> on visible pairs, p_ij = softmax_j(s_ij) and
+    o_i = sum_j p_ij v_j, the chain rule gives
+        dv_j = sum_i p_ij do_i
+        dp_ij = <do_i, v_j>
+        ds_ij = p_ij (dp_ij - sum_j' p_ij' dp_ij')
+        dq_i = scale sum_j ds_ij k_j,   dk_j = scale sum_i ds_ij q_i.
+    """
+    B, L, H, d = q.shape
+    mask = token_mask(L // tokens_per_frame, tokens_per_frame,
+                      frames_per_chunk, window)
+    dq = np.zeros_like(q)
+    dk = np.zeros_like(k)
+    dv = np.zeros_like(v)
+    for b in range(B):
+        for h in range(H):
+            p = softmax_rows(q[b, :, h], k[b, :, h], scale, mask)
+            dv[b, :, h] = p.T @ do[b, :, h]
+            dp = do[b, :, h] @ v[b, :, h].T
+            ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+            dq[b, :, h] = scale * ds @ k[b, :, h]
+            dk[b, :, h] = scale * ds.T @ q[b, :, h]
+    return dq, dk, dv

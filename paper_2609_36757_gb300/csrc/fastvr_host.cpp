@@ -389,6 +389,29 @@ fastvr_status_t fastvr_blockcausal_attn_fwd(const fastvr_attn_config_t* cfg,
   return FASTVR_OK;
 }
 
+fastvr_status_t fastvr_one_step_update(const void* z_lq, const void* v,
+                                       void* z_hat, int64_t n, float sigma,
+                                       int32_t dtype,
+                                       struct CUstream_st* stream) {
+  if (z_lq == nullptr || v == nullptr || z_hat == nullptr || n < 0 ||
+      !isfinite(sigma) || (dtype != 0 && dtype != 1) || !aligned16(z_lq) ||
+      !aligned16(v) || !aligned16(z_hat))
+    return FASTVR_ERR_INVALID_ARG;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) !=
+          cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  if (major != 10 || minor != 3) return FASTVR_ERR_UNSUPPORTED;
+  if (fastvr::launch_one_step(z_lq, v, z_hat, n, sigma, dtype,
+                              reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  return FASTVR_OK;
+}
+
 fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t p, int64_t* launches) {
   if (p == nullptr || launches == nullptr) return FASTVR_ERR_INVALID_ARG;
   *launches = p->launches;

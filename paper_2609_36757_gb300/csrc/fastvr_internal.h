@@ -65,6 +65,11 @@ struct AttnParams {
 };
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream);
+// The one-step update z_hat = z - sigma * v over n elements; z and out are
+// bf16 (dtype 0) or float32 (dtype 1), v is bf16.
+cudaError_t launch_one_step(const void* z, const void* v, void* out, int64_t n,
+                            float sigma, int dtype, cudaStream_t stream);
+
 // One-shot (training-form) attention over a whole token-major sequence.
 struct OneShotParams {
   const uint16_t* q;      // bfloat16 [B, L, H, d] token-major
@@ -80,6 +85,17 @@ struct OneShotParams {
   int* status;            // control word or null (timeouts not reported)
 };
 cudaError_t launch_blockcausal_attn(const OneShotParams& p, cudaStream_t stream);
+
+// Backward of the one-shot attention.
+struct BwdArgs {
+  const uint16_t *q, *k, *v, *out, *dout;  // bf16 [B, L, H, d] token-major
+  const float* lse;                        // forward LSE [B, H, L]
+  uint16_t *dq, *dk, *dv;                  // bf16 [B, L, H, d]
+  float* scratch;  // 2 * B * H * round_up(L, 128) floats
+  int32_t batch, heads, head_dim, seq_tokens, chunk_tokens, window;
+  float scale;
+};
+cudaError_t launch_blockcausal_attn_bwd(const BwdArgs& a, cudaStream_t stream);
 
 // Workspace parts (partial results) a launch of p uses on the current device
 // (0 when no unit is split), with at most kMaxParts parts.

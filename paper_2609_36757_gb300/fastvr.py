@@ -57,6 +57,8 @@ SIGNATURES = {
                                    ctypes.POINTER(_I64),
                                    ctypes.POINTER(_I64)]),
     "fastvr_plan_launch_count": (_I32, [_VP, ctypes.POINTER(_I64)]),
+    "fastvr_one_step_update": (_I32, [_VP, _VP, _VP, _I64, ctypes.c_float,
+                                      _I32, _VP]),
     "fastvr_blockcausal_attn_fwd": (_I32, [_CFGP, _I32, _VP, _VP, _VP, _VP,
                                            _VP, _VP]),
     "fastvr_chunk_attn_fwd_static": (_I32, [_CFGP, _VP, _I32, _VP, _VP, _I64,
@@ -202,6 +204,31 @@ def blockcausal_attention(cfg: fastvr_attn_config_t, q, k, v,
                                 0 if lse is None else lse.data_ptr(),
                                 torch.cuda.current_stream().cuda_stream)
     return (out, lse) if want_lse else out
+
+
+def fastvr_one_step_update(z_lq: int, v: int, z_hat: int, n: int,
+                           sigma: float, dtype: int, stream: int) -> None:
+    _check(lib.fastvr_one_step_update(z_lq, v, z_hat, n, sigma, dtype, stream),
+           "fastvr_one_step_update")
+
+
+def one_step_update(z_lq, v, sigma: float, out=None):
+    """Torch convenience: z_lq bfloat16 or float32, v bfloat16, same shape,
+    contiguous CUDA tensors; returns z_lq - sigma * v (in place when
+    out is z_lq)."""
+    import torch
+    if v.dtype != torch.bfloat16 or z_lq.dtype not in (torch.bfloat16,
+                                                       torch.float32):
+        raise ValueError("z_lq must be bfloat16 or float32 and v bfloat16")
+    if z_lq.shape != v.shape or not (z_lq.is_contiguous() and v.is_contiguous()):
+        raise ValueError("z_lq and v must be contiguous and of one shape")
+    if out is None:
+        out = torch.empty_like(z_lq)
+    fastvr_one_step_update(z_lq.data_ptr(), v.data_ptr(), out.data_ptr(),
+                           z_lq.numel(), sigma,
+                           0 if z_lq.dtype == torch.bfloat16 else 1,
+                           torch.cuda.current_stream().cuda_stream)
+    return out
 
 
 def fastvr_plan_launch_count(plan: int) -> int:

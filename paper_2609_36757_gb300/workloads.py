@@ -76,8 +76,21 @@ W1080P = Workload("1080p", 1, 12, 128, 68 * 120, 2, 15, seed=3)
 W1080P_WINDOWED = Workload("1080p-windowed", 1, 24, 128, 68 * 120, 3, 40,
                            window_chunks=4, last_chunk_frames=1, seed=4)
 
+# The paper's own inference shape (Sec. 4.1 "Inference"): chunks of k = 3
+# latent frames, each chunk sees itself and one predecessor (Eq. 1, W = 1),
+# and the frame is cut into overlapping 64 x 64 latent tiles, one DiT pass per
+# tile, so the tiles of a frame batch on B.  A 1080p frame (68 x 120 latent)
+# with tile stride 32 gives 2 x 3 = 6 tiles; 30 latent frames as above.  The DiT patch size is not
+# stated: a 2 x 2 patch gives 32 x 32 tokens per tile frame, none gives
+# 64 x 64.  Heads and head dim follow a 3072-wide DiT with 24 heads of 128.
+PAPER_TILES_32 = Workload("paper-tiles-32x32", 6, 24, 128, 32 * 32, 3, 10,
+                          window_chunks=1, seed=5)
+PAPER_TILES_64 = Workload("paper-tiles-64x64", 6, 24, 128, 64 * 64, 3, 10,
+                          window_chunks=1, seed=6)
+
 WORKLOADS = {w.name: w for w in
-             (TINY, W480P, W720P_PEAKED, W1080P, W1080P_WINDOWED)}
+             (TINY, W480P, W720P_PEAKED, W1080P, W1080P_WINDOWED,
+              PAPER_TILES_32, PAPER_TILES_64)}
 
 
 def chunk_stream(w: Workload) -> Iterator[Tuple[int, torch.Tensor, torch.Tensor,

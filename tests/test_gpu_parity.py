@@ -157,3 +157,13 @@ def test_paper_window_eq1_k3_w1_sampled_rows():
                   tokens_per_frame=8160, frames_per_chunk=3, num_chunks=5,
                   window_chunks=1, last_chunk_frames=2, seed=31)
     run_stream(w, rows_per_chunk=32).check()
+
+
+# ------------------------------------------- the paper's own inference shape
+def test_paper_tiles_32x32_sampled_rows():
+    # k = 3, W = 1, six overlapping 64 x 64 latent tiles batched on B
+    run_stream(WL.PAPER_TILES_32, rows_per_chunk=24, chunk_stride=3).check()
+
+
+def test_paper_tiles_64x64_sampled_rows():
+    run_stream(WL.PAPER_TILES_64, rows_per_chunk=16, chunk_stride=3).check()
