@@ -168,6 +168,31 @@ FASTVR_API fastvr_status_t fastvr_blockcausal_attn_fwd(
     const void* k, const void* v, void* out, float* lse,
     struct CUstream_st* stream);
 
+/* Scratch bytes fastvr_blockcausal_attn_bwd needs for cfg and num_frames:
+ * 2 * B * H * round_up(L, 128) floats (per-row log-sum-exp and D).  Host only.
+ * Errors: INVALID_ARG, UNSUPPORTED. */
+FASTVR_API fastvr_status_t fastvr_blockcausal_bwd_scratch_bytes(
+    const fastvr_attn_config_t* cfg, int32_t num_frames, size_t* bytes);
+
+/* Gradients of the one-shot chunk-causal attention (the training form of
+ * Sec. 3.1; the paper trains the DiT under the mask M of Eq. 1).  Inputs:
+ * q, k, v, out (the forward output) and dout (its gradient), bfloat16
+ * [B, L, H, d] token-major; lse, float32 [B, H, L], the forward's
+ * log-sum-exp (fastvr_blockcausal_attn_fwd).  Outputs dq, dk, dv bfloat16
+ * [B, L, H, d].  scratch: caller-owned device memory of at least
+ * fastvr_blockcausal_bwd_scratch_bytes bytes, overwritten.  Computes
+ * D = rowsum(dout * out), then dk/dv (one CTA per 128 keys, over the query
+ * tiles that see them) and dq (one CTA per 128 queries); P is recomputed
+ * from lse, P and dS enter the tensor cores in bfloat16, accumulation is
+ * fp32.  All pointers 16-byte aligned.  A bounded-wait timeout leaves the
+ * outputs undefined and is not reported.
+ * Errors: INVALID_ARG, UNSUPPORTED, CAPACITY (scratch too small), CUDA. */
+FASTVR_API fastvr_status_t fastvr_blockcausal_attn_bwd(
+    const fastvr_attn_config_t* cfg, int32_t num_frames, const void* q,
+    const void* k, const void* v, const void* out, const void* dout,
+    const float* lse, void* dq, void* dk, void* dv, float* scratch,
+    size_t scratch_bytes, struct CUstream_st* stream);
+
 /* FastVR's one-step restoration update (Eq. `eq:one_step`, used at
  * inference and in Stage II training): z_hat = z_lq - sigma * v, with v the
  * DiT's predicted velocity at t = tau and sigma = sigma_tau (an input: the

@@ -22,7 +22,7 @@ LIB = os.path.join(HERE, "libfastvr_attn.so")
 INCLUDE = os.path.join(ROOT, "include")
 
 SOURCES = ["fastvr_host.cpp", "kv_append.cu", "chunk_attn_fwd.cu",
-           "chunk_attn_static.cu", "one_step.cu"]
+           "chunk_attn_static.cu", "one_step.cu", "chunk_attn_bwd.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",
          "-Xcompiler", "-fvisibility=hidden", "-I", INCLUDE, "-I", CSRC]

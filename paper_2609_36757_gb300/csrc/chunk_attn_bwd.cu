@@ -1,0 +1,634 @@
+// Backward of one-shot chunk-causal attention (the training form of
+// Sec. 3.1: the whole latent sequence at once under the mask of Eq. 1),
+// with tcgen05 tensor cores, TMEM accumulators and TMA-staged tiles.
+//
+// With s_ij = scale <q_i, k_j> on visible pairs, P = softmax(S) (row i,
+// recomputed from the forward's log-sum-exp), dO the output gradient and
+// D_i = <dO_i, O_i>:
+//     dV = P^T dO,  dP = dO V^T,  dS = P o (dP - D),
+//     dQ = scale dS K,  dK = scale dS^T Q.
+// Three kernels, no atomics:
+//   delta_kernel  D_i = <dO_i, O_i> (fp32) into the caller's scratch;
+//   dkdv_kernel   one CTA per 128-key tile: for every query tile that sees it
+//                 S^T = K Q^T and dP^T = V dO^T (SMEM x SMEM -> TMEM), then
+//                 P^T and dS^T in bf16 over them in TMEM, then
+//                 dV += P^T dO and dK += dS^T Q (A from TMEM, B = dO or Q
+//                 read as an MN-major operand);
+//   dq_kernel     one CTA per 128-query tile: for every visible key tile
+//                 S = Q K^T, dP = dO V^T, dS, dQ += dS K.
+// Visibility is Eq. 1 with window W per (query row, key): a key of chunk c'
+// is seen by queries of chunks c' .. c' + W, a query of chunk c sees keys of
+// chunks c - W .. c; only tiles inside a CTA's visible range are loaded and
+// columns outside each row's range are masked.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+
+#include "fastvr_internal.h"
+#include "sm100_ptx.cuh"
+
+namespace fastvr {
+namespace {
+
+using namespace sm100;
+
+constexpr int kT = 128;           // tile rows (TMEM lanes) and tile columns
+constexpr int kBox = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (bytes)
+constexpr int kStages = 2;        // streamed-operand ring depth
+constexpr int kThreads = 192;     // 4 compute warps, producer, MMA issuer
+constexpr uint32_t kTmemCols = 512;
+constexpr uint64_t kWaitLimitNs = 4000000000ull;
+
+struct BwdParams {
+  CUtensorMap q_map, k_map, v_map, do_map;  // {d, L, H, B} token-major
+  const float* lse2;   // forward LSE in log2 units [B*H, Lpad] (scratch)
+  const float* delta;  // D [B*H, Lpad] (scratch); padding tokens hold 0
+  uint16_t* dq;        // bf16 [B, L, H, d]
+  uint16_t* dk;
+  uint16_t* dv;
+  int32_t seq_tokens, heads, batch, chunk_tokens, window, tiles, padded;
+  float scale, scale_log2;
+};
+
+struct BwdShared {
+  uint64_t fixed_full;                 // the CTA's resident operands
+  uint64_t full[kStages], empty[kStages];
+  uint64_t s_full, p_full, o_full, drain;
+  uint32_t tmem_base;
+  int abort;
+  // dkdv: the streamed query tile's log2 LSE and D, one slice per stage
+  __align__(16) float lse2[kStages][kT];
+  __align__(16) float dlt[kStages][kT];
+};
+
+template <int D>
+struct BwdLayout {
+  static constexpr int kNB = D / 64;
+  // fixed operands (two tiles), then the streamed ring of two tiles a stage
+  __host__ __device__ static constexpr int fixed(int which, int bx) {
+    return (which * kNB + bx) * kBox;
+  }
+  __host__ __device__ static constexpr int ring(int st, int which, int bx) {
+    return ((2 + st * 2 + which) * kNB + bx) * kBox;
+  }
+  static constexpr int shared_off = (2 + 2 * kStages) * kNB * kBox;
+  static constexpr int bytes = shared_off + (int)sizeof(BwdShared) + 1024 + 64;
+};
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
+                                         BwdShared* S) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*reinterpret_cast<volatile int*>(&S->abort)) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      *reinterpret_cast<volatile int*>(&S->abort) = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (global_timer_ns() - t0 > kWaitLimitNs) return;
+}
+
+// Row of the padded [B*H, Lpad] scratch vectors.
+__device__ __forceinline__ int bh_row(const BwdParams& p, int b, int h) {
+  return b * p.heads + h;
+}
+
+// Visible query tokens of a key in chunk c (Eq. 1 read from the key side).
+__device__ __forceinline__ void key_sees(const BwdParams& p, int key, int& lo,
+                                         int& hi) {
+  if (key >= p.seq_tokens) {
+    lo = hi = 0;
+    return;
+  }
+  const int c = key / p.chunk_tokens;
+  lo = c * p.chunk_tokens;
+  hi = p.window < 0 ? p.seq_tokens
+                    : min((c + p.window + 1) * p.chunk_tokens, p.seq_tokens);
+}
+
+// Visible key tokens of a query in chunk c.
+__device__ __forceinline__ void query_sees(const BwdParams& p, int row, int& lo,
+                                           int& hi) {
+  const int c = min(row, p.seq_tokens - 1) / p.chunk_tokens;
+  lo = p.window < 0 ? 0 : max(0, c - p.window) * p.chunk_tokens;
+  hi = min((c + 1) * p.chunk_tokens, p.seq_tokens);
+}
+
+// Common CTA prologue: TMEM (warp 5) and barriers (thread 128).
+__device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
+  const int warp = threadIdx.x / 32;
+  if (warp == 5) {
+    tmem_alloc(&S->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  if (threadIdx.x == 128) {
+    mbar_init(&S->fixed_full, 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&S->full[s], 1);
+      mbar_init(&S->empty[s], 1);
+    }
+    mbar_init(&S->s_full, 1);
+    mbar_init(&S->p_full, 4 * 32);
+    mbar_init(&S->o_full, 1);
+    mbar_init(&S->drain, 1);
+    S->abort = 0;
+    fence_barrier_init();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  return S->tmem_base;
+}
+
+__device__ __forceinline__ void bwd_teardown(uint32_t tmem) {
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x / 32 == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// Producer: two resident tiles (maps f0, f1 at token t_fixed), then two
+// streamed tiles per step (maps r0, r1 at token t0 + 128 j).
+// With kRowVecs, each step also bulk-copies the streamed tile's 128 log2-LSE
+// and D values (from the padded scratch rows vec_lse2, vec_dlt).
+template <int D, bool kRowVecs>
+__device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
+                             const CUtensorMap* f1, int t_fixed,
+                             const CUtensorMap* r0, const CUtensorMap* r1,
+                             int t0, int n, int h, int b,
+                             const float* vec_lse2, const float* vec_dlt) {
+  using L = BwdLayout<D>;
+  constexpr uint32_t kVecBytes = kRowVecs ? 2 * kT * sizeof(float) : 0;
+  mbar_arrive_expect_tx(&S->fixed_full, 2 * L::kNB * kBox);
+  for (int bx = 0; bx < L::kNB; ++bx) {
+    tma_load_4d(f0, smem + L::fixed(0, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
+    tma_load_4d(f1, smem + L::fixed(1, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
+  }
+  int issued = 0;
+  for (int j = 0; j < n; ++j) {
+    const int st = j % kStages;
+    if (!wait_bar(&S->empty[st], ((j / kStages) & 1) ^ 1, S)) break;
+    mbar_arrive_expect_tx(&S->full[st], 2 * L::kNB * kBox + kVecBytes);
+    for (int bx = 0; bx < L::kNB; ++bx) {
+      tma_load_4d(r0, smem + L::ring(st, 0, bx), &S->full[st], bx * 64,
+                  t0 + j * kT, h, b);
+      tma_load_4d(r1, smem + L::ring(st, 1, bx), &S->full[st], bx * 64,
+                  t0 + j * kT, h, b);
+    }
+    if (kRowVecs) {
+      bulk_load(S->lse2[st], vec_lse2 + t0 + j * kT, kT * sizeof(float),
+                &S->full[st]);
+      bulk_load(S->dlt[st], vec_dlt + t0 + j * kT, kT * sizeof(float),
+                &S->full[st]);
+    }
+    ++issued;
+  }
+  drain_wait(&S->fixed_full, 0);
+  for (int i = max(0, issued - kStages); i < issued; ++i)
+    drain_wait(&S->full[i % kStages], (i / kStages) & 1);
+}
+
+// D_t = A_fixed * B_ring^T over the head dim (both K-major): TMEM col c0.
+template <int D>
+__device__ __forceinline__ void mma_nt(uint32_t sbase, uint32_t tmem, int c0,
+                                       int fixed_which, int st, int ring_which) {
+  using L = BwdLayout<D>;
+  constexpr uint32_t kIdesc = idesc_bf16_f32(kT, kT, 0);
+#pragma unroll
+  for (int ks = 0; ks < D / 16; ++ks) {
+    const uint32_t off = (ks / 4) * kBox + (ks % 4) * 32;
+    mma_ss(tmem + c0,
+           smem_desc_sw128(sbase + L::fixed(fixed_which, 0) + off, 16, 1024),
+           smem_desc_sw128(sbase + L::ring(st, ring_which, 0) + off, 16, 1024),
+           kIdesc, ks > 0);
+  }
+}
+
+// D (+)= A_tmem (128 x 128, bf16 pairs at column a0) * B, B an MN-major
+// [128 x d] tile at SMEM offset b_off: TMEM column c0.
+template <int D>
+__device__ __forceinline__ void mma_tn(uint32_t sbase, uint32_t tmem, int c0,
+                                       int a0, int b_off, int acc) {
+  constexpr uint32_t kIdesc = idesc_bf16_f32(kT, D, 1);
+#pragma unroll
+  for (int kk = 0; kk < kT / 16; ++kk)
+    mma_ts(tmem + c0, tmem + a0 + kk * 8,
+           smem_desc_sw128(sbase + b_off + kk * 2048, kBox, 1024), kIdesc,
+           (acc | kk) != 0);
+}
+
+// Write 32 fp32 accumulator columns (scaled) of a TMEM row as bf16.
+__device__ __forceinline__ void store_row32(uint32_t taddr, float mul,
+                                            uint16_t* dst, bool ok) {
+  uint32_t r[32];
+  tmem_ld32(taddr, r);
+  tmem_wait_ld();
+  uint32_t pk[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    pk[i] = pack_bf16(__uint_as_float(r[2 * i]) * mul,
+                      __uint_as_float(r[2 * i + 1]) * mul);
+  if (ok) {
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+    for (int v = 0; v < 4; ++v)
+      d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+  }
+}
+
+// ------------------------------------------------------------------ dK, dV
+// TMEM: [0,128) S^T then P^T (bf16, first 64 columns), [128,256) dP^T then
+// dS^T, [256,256+d) dV, [384,384+d) dK.  Resident: K (fixed 0), V (fixed 1).
+// Streamed: Q (ring 0), dO (ring 1).
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+dkdv_kernel(const __grid_constant__ BwdParams p) {
+  using L = BwdLayout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  BwdShared* S = reinterpret_cast<BwdShared*>(smem + L::shared_off);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int bh = blockIdx.x % (p.heads * p.batch);
+  const int h = bh % p.heads, b = bh / p.heads;
+  const int k0 = (blockIdx.x / (p.heads * p.batch)) * kT;  // first key
+  // Queries that see any key of the tile: chunks c(k0) .. c(k_last) + W.
+  const int k_last = min(k0 + kT, p.seq_tokens) - 1;
+  // Query tiles start at a multiple of 128 at or below the first visible
+  // query (rows before it are masked), so each tile's 128 log2-LSE and D
+  // values are one aligned slice inside the padded scratch row.
+  const int q0 = (k0 / p.chunk_tokens) * p.chunk_tokens / kT * kT;
+  const int q1 = p.window < 0 ? p.seq_tokens
+                              : min((k_last / p.chunk_tokens + p.window + 1) *
+                                        p.chunk_tokens,
+                                    p.seq_tokens);
+  const int n = (q1 - q0 + kT - 1) / kT;
+  const uint32_t tmem = bwd_setup(S);
+
+  if (warp == 4) {
+    if (lane == 0)
+      bwd_producer<D, true>(smem, S, &p.k_map, &p.v_map, k0, &p.q_map,
+                            &p.do_map, q0, n, h, b,
+                            p.lse2 + (int64_t)bh_row(p, b, h) * p.padded,
+                            p.delta + (int64_t)bh_row(p, b, h) * p.padded);
+    __syncwarp();
+  } else if (warp == 5) {
+    if (lane == 0) {
+      const uint32_t sbase = smem_addr(smem);
+      bool ok = wait_bar(&S->fixed_full, 0, S);
+      for (int j = 0; ok && j < n; ++j) {
+        const int st = j % kStages;
+        if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
+        tc_fence_after();
+        mma_nt<D>(sbase, tmem, 0, 0, st, 0);    // S^T = K Q^T
+        mma_nt<D>(sbase, tmem, 128, 1, st, 1);  // dP^T = V dO^T
+        mma_commit(&S->s_full);
+        if (!(ok = wait_bar(&S->p_full, j & 1, S))) break;
+        tc_fence_after();
+        mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
+        mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
+        mma_commit(&S->empty[st]);
+      }
+      if (ok) mma_commit(&S->o_full);
+      mma_commit(&S->drain);
+      drain_wait(&S->drain, 0);
+    }
+    __syncwarp();
+  } else {
+    // Compute warps: thread = key row (TMEM lane) of the tile.
+    const int t = threadIdx.x;  // 0..127
+    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    int vis_lo, vis_hi;
+    key_sees(p, k0 + t, vis_lo, vis_hi);
+    const float c2 = p.scale_log2;
+    bool ok = true;
+    for (int j = 0; j < n; ++j) {
+      const int i0 = q0 + j * kT;  // first query of the tile
+      const int st = j % kStages;
+      // the stage's LSE and D slices (the MMA warp frees the stage only after
+      // p_full, so they stay valid while this tile is processed)
+      if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
+      if (!(ok = wait_bar(&S->s_full, j & 1, S))) break;
+      tc_fence_after();
+      const float* lse2 = S->lse2[st];
+      const float* dlt = S->dlt[st];
+      const int lo = vis_lo - i0, hi = vis_hi - i0;
+      const bool need_mask = lo > 0 || hi < kT;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {  // 32 query columns at a time
+        uint32_t s[32], dp[32];
+        tmem_ld32(tmem + lane_off + c * 32, s);
+        tmem_ld32(tmem + lane_off + 128 + c * 32, dp);
+        tmem_wait_ld();
+        uint32_t pp[16], pd[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          float pv[2], dv[2];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int col = c * 32 + 2 * e + u;
+            float x = fmaf(__uint_as_float(s[2 * e + u]), c2, -lse2[col]);
+            if (need_mask && (col < lo || col >= hi)) x = -INFINITY;
+            pv[u] = ex2(x);
+            dv[u] = pv[u] * (__uint_as_float(dp[2 * e + u]) - dlt[col]);
+          }
+          pp[e] = pack_bf16(pv[0], pv[1]);
+          pd[e] = pack_bf16(dv[0], dv[1]);
+        }
+        tmem_st16(tmem + lane_off + c * 16, pp);        // P^T over S^T
+        tmem_st16(tmem + lane_off + 128 + c * 16, pd);  // dS^T over dP^T
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&S->p_full);
+    }
+    if (ok && wait_bar(&S->o_full, 0, S)) {
+      tc_fence_after();
+      const int key = k0 + t;
+      const bool in_range = key < p.seq_tokens;
+      const int64_t off = (int64_t)b * p.seq_tokens * p.heads * D +
+                          (int64_t)(in_range ? key : 0) * p.heads * D +
+                          (int64_t)h * D;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        store_row32(tmem + lane_off + 256 + c * 32, 1.f, p.dv + off + c * 32,
+                    in_range);
+        store_row32(tmem + lane_off + 384 + c * 32, p.scale, p.dk + off + c * 32,
+                    in_range);
+      }
+    }
+  }
+  bwd_teardown(tmem);
+}
+
+// --------------------------------------------------------------------- dQ
+// TMEM: [0,128) S, [128,256) dP then dS (bf16, first 64 columns),
+// [256,256+d) dQ.  Resident: Q (fixed 0), dO (fixed 1).  Streamed: K (ring
+// 0), V (ring 1).
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+dq_kernel(const __grid_constant__ BwdParams p) {
+  using L = BwdLayout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  BwdShared* S = reinterpret_cast<BwdShared*>(smem + L::shared_off);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int bh = blockIdx.x % (p.heads * p.batch);
+  const int h = bh % p.heads, b = bh / p.heads;
+  // longest key ranges first
+  const int q0 = (p.tiles - 1 - blockIdx.x / (p.heads * p.batch)) * kT;
+  const int q_last = min(q0 + kT, p.seq_tokens) - 1;
+  const int c_lo = q0 / p.chunk_tokens, c_hi = q_last / p.chunk_tokens;
+  const int kv0 = p.window < 0 ? 0 : max(0, c_lo - p.window) * p.chunk_tokens;
+  const int kv1 = min((c_hi + 1) * p.chunk_tokens, p.seq_tokens);
+  const int n = (kv1 - kv0 + kT - 1) / kT;
+  const uint32_t tmem = bwd_setup(S);
+
+  if (warp == 4) {
+    if (lane == 0)
+      bwd_producer<D, false>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map,
+                             &p.v_map, kv0, n, h, b, nullptr, nullptr);
+    __syncwarp();
+  } else if (warp == 5) {
+    if (lane == 0) {
+      const uint32_t sbase = smem_addr(smem);
+      bool ok = wait_bar(&S->fixed_full, 0, S);
+      for (int j = 0; ok && j < n; ++j) {
+        const int st = j % kStages;
+        if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
+        tc_fence_after();
+        mma_nt<D>(sbase, tmem, 0, 0, st, 0);    // S = Q K^T
+        mma_nt<D>(sbase, tmem, 128, 1, st, 1);  // dP = dO V^T
+        mma_commit(&S->s_full);
+        if (!(ok = wait_bar(&S->p_full, j & 1, S))) break;
+        tc_fence_after();
+        mma_tn<D>(sbase, tmem, 256, 128, L::ring(st, 0, 0), j > 0);  // dQ
+        mma_commit(&S->empty[st]);
+      }
+      if (ok) mma_commit(&S->o_full);
+      mma_commit(&S->drain);
+      drain_wait(&S->drain, 0);
+    }
+    __syncwarp();
+  } else {
+    // Compute warps: thread = query row (TMEM lane).
+    const int t = threadIdx.x;
+    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    const int row = q0 + t;
+    const bool in_range = row < p.seq_tokens;
+    int vis_lo, vis_hi;
+    query_sees(p, row, vis_lo, vis_hi);
+    const int64_t rl = (int64_t)bh_row(p, b, h) * p.padded + row;
+    const float lse2 = p.lse2[rl];  // the padded rows hold 0
+    const float dlt = p.delta[rl];
+    const float c2 = p.scale_log2;
+    bool ok = true;
+    for (int j = 0; j < n; ++j) {
+      const int tok0 = kv0 + j * kT;
+      if (!(ok = wait_bar(&S->s_full, j & 1, S))) break;
+      tc_fence_after();
+      const int lo = vis_lo - tok0;
+      const int hi = min(vis_hi, kv1) - tok0;
+      const bool need_mask = lo > 0 || hi < kT || !in_range;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t s[32], dp[32];
+        tmem_ld32(tmem + lane_off + c * 32, s);
+        tmem_ld32(tmem + lane_off + 128 + c * 32, dp);
+        tmem_wait_ld();
+        uint32_t pd[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          float dv[2];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int col = c * 32 + 2 * e + u;
+            float x = fmaf(__uint_as_float(s[2 * e + u]), c2, -lse2);
+            if (need_mask && (col < lo || col >= hi || !in_range)) x = -INFINITY;
+            dv[u] = ex2(x) * (__uint_as_float(dp[2 * e + u]) - dlt);
+          }
+          pd[e] = pack_bf16(dv[0], dv[1]);
+        }
+        tmem_st16(tmem + lane_off + 128 + c * 16, pd);  // dS over dP
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&S->p_full);
+    }
+    if (ok && wait_bar(&S->o_full, 0, S)) {
+      tc_fence_after();
+      const int64_t off = (int64_t)b * p.seq_tokens * p.heads * D +
+                          (int64_t)(in_range ? row : 0) * p.heads * D +
+                          (int64_t)h * D;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c)
+        store_row32(tmem + lane_off + 256 + c * 32, p.scale, p.dq + off + c * 32,
+                    in_range);
+    }
+  }
+  bwd_teardown(tmem);
+}
+
+// Scratch rows for the backward: D_i = <dO_i, O_i> over the head dim and
+// the forward LSE in log2 units, each [B*H, Lpad] with Lpad = L rounded up to
+// 128 and zeros in the padding (so every 128-token slice is aligned and in
+// bounds).  One warp per (b, token, head) row of O.
+template <int D>
+__global__ void __launch_bounds__(256)
+delta_kernel(const uint16_t* o, const uint16_t* dO, const float* lse,
+             float* lse2, float* delta, int batch, int heads, int seq,
+             int padded) {
+  const int64_t rows = (int64_t)batch * seq * heads;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
+  const int lane = threadIdx.x % 32;
+  const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
+  for (int64_t r = warp; r < rows; r += nwarps) {  // r = (b, token, head)
+    float acc = 0.f;
+    for (int x = lane * 2; x < D; x += 64) {
+      const __nv_bfloat162 a =
+          *reinterpret_cast<const __nv_bfloat162*>(o + r * D + x);
+      const __nv_bfloat162 g =
+          *reinterpret_cast<const __nv_bfloat162*>(dO + r * D + x);
+      acc = fmaf(__low2float(a), __low2float(g), acc);
+      acc = fmaf(__high2float(a), __high2float(g), acc);
+    }
+#pragma unroll
+    for (int m = 16; m > 0; m >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, m);
+    if (lane == 0) {
+      const int64_t h = r % heads, bt = r / heads;
+      const int64_t tok = bt % seq, b = bt / seq;
+      const int64_t i = (b * heads + h) * padded + tok;
+      delta[i] = acc;
+      lse2[i] = lse[(b * heads + h) * seq + tok] * 1.4426950408889634f;
+    }
+  }
+  // padding tokens
+  const int64_t pad = padded - seq;
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (int64_t i = tid; i < (int64_t)batch * heads * pad;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t j = (i / pad) * padded + seq + i % pad;
+    delta[j] = 0.f;
+    lse2[j] = 0.f;
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType,
+                                  cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (fn == nullptr) {
+    cudaDriverEntryPointQueryResult q;
+    void* ptr = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// Token-major [B, L, H, d] bf16 tensor as a 4-D map over (d, token, head,
+// batch), box 64 x 128, 128-byte swizzle; tokens past L read as zeros.
+bool token_major_map(CUtensorMap* m, const void* base, int d, int L, int H,
+                     int B) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  const cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)L, (cuuint64_t)H,
+                              (cuuint64_t)B};
+  const cuuint64_t strides[3] = {(cuuint64_t)H * d * 2, (cuuint64_t)d * 2,
+                                 (cuuint64_t)L * H * d * 2};
+  const cuuint32_t box[4] = {64, 128, 1, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base),
+             dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
+  BwdParams p;
+  memset(&p, 0, sizeof(p));
+  const int L = a.seq_tokens;
+  if (!token_major_map(&p.q_map, a.q, D, L, a.heads, a.batch) ||
+      !token_major_map(&p.k_map, a.k, D, L, a.heads, a.batch) ||
+      !token_major_map(&p.v_map, a.v, D, L, a.heads, a.batch) ||
+      !token_major_map(&p.do_map, a.dout, D, L, a.heads, a.batch))
+    return cudaErrorInvalidValue;
+  const int padded = (L + kT - 1) / kT * kT;
+  p.lse2 = a.scratch;
+  p.delta = a.scratch + (size_t)a.batch * a.heads * padded;
+  p.padded = padded;
+  p.dq = a.dq;
+  p.dk = a.dk;
+  p.dv = a.dv;
+  p.seq_tokens = L;
+  p.heads = a.heads;
+  p.batch = a.batch;
+  p.chunk_tokens = a.chunk_tokens;
+  p.window = a.window;
+  p.tiles = (L + kT - 1) / kT;
+  p.scale = a.scale;
+  p.scale_log2 = a.scale * 1.4426950408889634f;
+
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t rows = (int64_t)a.batch * L * a.heads;
+  int64_t blocks = std::min<int64_t>((int64_t)(sms > 0 ? sms : 152) * 8,
+                                     (rows + 7) / 8);
+  delta_kernel<D><<<(unsigned)blocks, 256, 0, stream>>>(
+      a.out, a.dout, a.lse, a.scratch, a.scratch + (size_t)a.batch * a.heads * padded,
+      a.batch, a.heads, L, padded);
+  const int smem = BwdLayout<D>::bytes;
+  cudaError_t e = cudaFuncSetAttribute(
+      dkdv_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(dq_kernel<D>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const int grid = p.tiles * a.heads * a.batch;
+  dkdv_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+  dq_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_blockcausal_attn_bwd(const BwdArgs& a, cudaStream_t stream) {
+  if (a.head_dim == 64) return launch_bwd_d<64>(a, stream);
+  if (a.head_dim == 128) return launch_bwd_d<128>(a, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace fastvr

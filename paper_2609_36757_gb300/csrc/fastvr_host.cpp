@@ -389,6 +389,82 @@ fastvr_status_t fastvr_blockcausal_attn_fwd(const fastvr_attn_config_t* cfg,
   return FASTVR_OK;
 }
 
+namespace {
+// Validation shared by the one-shot backward entry points.
+fastvr_status_t check_oneshot_cfg(const fastvr_attn_config_t* cfg,
+                                  int32_t num_frames) {
+  if (cfg == nullptr || cfg->batch < 1 || cfg->heads < 1 ||
+      cfg->tokens_per_frame < 1 || cfg->frames_per_chunk < 1 ||
+      cfg->window_chunks < -1 || !(cfg->softmax_scale >= 0.f) ||
+      !isfinite(cfg->softmax_scale) || num_frames < 1)
+    return FASTVR_ERR_INVALID_ARG;
+  if (!supported_dim(cfg->head_dim)) return FASTVR_ERR_UNSUPPORTED;
+  const int64_t L = (int64_t)num_frames * cfg->tokens_per_frame;
+  if (L > INT32_MAX / 2 ||
+      (int64_t)cfg->frames_per_chunk * cfg->tokens_per_frame > INT32_MAX / 2)
+    return FASTVR_ERR_INVALID_ARG;
+  return FASTVR_OK;
+}
+}  // namespace
+
+fastvr_status_t fastvr_blockcausal_bwd_scratch_bytes(
+    const fastvr_attn_config_t* cfg, int32_t num_frames, size_t* bytes) {
+  fastvr_status_t st = check_oneshot_cfg(cfg, num_frames);
+  if (st != FASTVR_OK) return st;
+  if (bytes == nullptr) return FASTVR_ERR_INVALID_ARG;
+  const int64_t L = (int64_t)num_frames * cfg->tokens_per_frame;
+  const int64_t padded = (L + 127) / 128 * 128;
+  *bytes = (size_t)(2 * (int64_t)cfg->batch * cfg->heads * padded * 4);
+  return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_blockcausal_attn_bwd(
+    const fastvr_attn_config_t* cfg, int32_t num_frames, const void* q,
+    const void* k, const void* v, const void* out, const void* dout,
+    const float* lse, void* dq, void* dk, void* dv, float* scratch,
+    size_t scratch_bytes, struct CUstream_st* stream) {
+  fastvr_status_t st = check_oneshot_cfg(cfg, num_frames);
+  if (st != FASTVR_OK) return st;
+  const void* ptrs[] = {q, k, v, out, dout, lse, dq, dk, dv, scratch};
+  for (const void* ptr : ptrs)
+    if (ptr == nullptr || !aligned16(ptr)) return FASTVR_ERR_INVALID_ARG;
+  size_t need = 0;
+  fastvr_blockcausal_bwd_scratch_bytes(cfg, num_frames, &need);
+  if (scratch_bytes < need) return FASTVR_ERR_CAPACITY;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) !=
+          cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  if (major != 10 || minor != 3) return FASTVR_ERR_UNSUPPORTED;
+  fastvr::BwdArgs a;
+  memset(&a, 0, sizeof(a));
+  a.q = static_cast<const uint16_t*>(q);
+  a.k = static_cast<const uint16_t*>(k);
+  a.v = static_cast<const uint16_t*>(v);
+  a.out = static_cast<const uint16_t*>(out);
+  a.dout = static_cast<const uint16_t*>(dout);
+  a.lse = lse;
+  a.dq = static_cast<uint16_t*>(dq);
+  a.dk = static_cast<uint16_t*>(dk);
+  a.dv = static_cast<uint16_t*>(dv);
+  a.scratch = scratch;
+  a.batch = cfg->batch;
+  a.heads = cfg->heads;
+  a.head_dim = cfg->head_dim;
+  a.seq_tokens = num_frames * cfg->tokens_per_frame;
+  a.chunk_tokens = cfg->frames_per_chunk * cfg->tokens_per_frame;
+  a.window = cfg->window_chunks;
+  a.scale = cfg->softmax_scale == 0.f ? 1.f / sqrtf((float)cfg->head_dim)
+                                      : cfg->softmax_scale;
+  if (fastvr::launch_blockcausal_attn_bwd(
+          a, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  return FASTVR_OK;
+}
+
 fastvr_status_t fastvr_one_step_update(const void* z_lq, const void* v,
                                        void* z_hat, int64_t n, float sigma,
                                        int32_t dtype,

@@ -59,6 +59,10 @@ SIGNATURES = {
     "fastvr_plan_launch_count": (_I32, [_VP, ctypes.POINTER(_I64)]),
     "fastvr_one_step_update": (_I32, [_VP, _VP, _VP, _I64, ctypes.c_float,
                                       _I32, _VP]),
+    "fastvr_blockcausal_bwd_scratch_bytes": (_I32, [_CFGP, _I32,
+                                                    ctypes.POINTER(_SZ)]),
+    "fastvr_blockcausal_attn_bwd": (_I32, [_CFGP, _I32] + [_VP] * 10 +
+                                    [_SZ, _VP]),
     "fastvr_blockcausal_attn_fwd": (_I32, [_CFGP, _I32, _VP, _VP, _VP, _VP,
                                            _VP, _VP]),
     "fastvr_chunk_attn_fwd_static": (_I32, [_CFGP, _VP, _I32, _VP, _VP, _I64,
@@ -204,6 +208,41 @@ def blockcausal_attention(cfg: fastvr_attn_config_t, q, k, v,
                                 0 if lse is None else lse.data_ptr(),
                                 torch.cuda.current_stream().cuda_stream)
     return (out, lse) if want_lse else out
+
+
+def fastvr_blockcausal_bwd_scratch_bytes(cfg: fastvr_attn_config_t,
+                                         num_frames: int) -> int:
+    n = _SZ(0)
+    _check(lib.fastvr_blockcausal_bwd_scratch_bytes(ctypes.byref(cfg),
+                                                    num_frames, ctypes.byref(n)),
+           "fastvr_blockcausal_bwd_scratch_bytes")
+    return n.value
+
+
+def fastvr_blockcausal_attn_bwd(cfg, num_frames, q, k, v, out, dout, lse, dq,
+                                dk, dv, scratch, scratch_bytes, stream) -> None:
+    _check(lib.fastvr_blockcausal_attn_bwd(
+        ctypes.byref(cfg), num_frames, q, k, v, out, dout, lse, dq, dk, dv,
+        scratch, scratch_bytes, stream), "fastvr_blockcausal_attn_bwd")
+
+
+def blockcausal_attention_bwd(cfg: fastvr_attn_config_t, q, k, v, out, dout,
+                              lse):
+    """Torch convenience for fastvr_blockcausal_attn_bwd: bfloat16 CUDA
+    tensors [B, L, H, d] and the forward's float32 lse [B, H, L]; returns
+    (dq, dk, dv).  The scratch is allocated with torch."""
+    import torch
+    L = q.shape[1]
+    frames = L // cfg.tokens_per_frame
+    nbytes = fastvr_blockcausal_bwd_scratch_bytes(cfg, frames)
+    scratch = torch.empty(nbytes // 4, dtype=torch.float32, device=q.device)
+    dq, dk, dv = (torch.empty_like(q) for _ in range(3))
+    fastvr_blockcausal_attn_bwd(
+        cfg, frames, q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+        dout.data_ptr(), lse.data_ptr(), dq.data_ptr(), dk.data_ptr(),
+        dv.data_ptr(), scratch.data_ptr(), nbytes,
+        torch.cuda.current_stream().cuda_stream)
+    return dq, dk, dv
 
 
 def fastvr_one_step_update(z_lq: int, v: int, z_hat: int, n: int,
