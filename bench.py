@@ -383,6 +383,73 @@ def measure_one_step(dev, sets: int = 8, rounds: int = 3):
             "l2": f"{sets} distinct latents rotated ({sets * 6 * n / 1e6:.0f} MB)"}
 
 
+def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
+    """One-shot (training) form over a whole sequence: forward, and in
+    `train` mode the backward too.  FLOPs: forward 4 B H d x visible pairs;
+    backward 2.5 x that (five products of the same size: S recomputed, dP,
+    dV, dQ, dK; the kernels compute two more to avoid atomics, not counted)."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = WORKLOAD
+    lk = visible_tokens_per_chunk(w)
+    fwd_flops = sum(chunk_flops(w, lk[c], c) for c in range(w.num_chunks))
+    chunks = host_chunks(w, seed_offset=rank)
+    q, k, v = (torch.cat([c[i] for c in chunks], 1).to(dev) for i in range(3))
+    do = torch.randn_like(q, dtype=torch.float32).to(torch.bfloat16)
+    cfg = FV.config_from_workload(w)
+    train = args.mode == "train"
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev):
+        ev[0].record(stream)
+        o, lse = FV.blockcausal_attention(cfg, q, k, v, want_lse=True)
+        ev[1].record(stream)
+        if train:
+            FV.blockcausal_attention_bwd(cfg, q, k, v, o, do, lse)
+        ev[2].record(stream)
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)]
+           for _ in range(args.warmup + args.steps)]
+    for i in range(args.warmup):
+        step(evs[i])
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    for i in range(args.warmup, args.warmup + args.steps):
+        step(evs[i])
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    timed = evs[args.warmup:]
+    fwd_ms = statistics.median(e[0].elapsed_time(e[1]) for e in timed)
+    bwd_ms = statistics.median(e[1].elapsed_time(e[2]) for e in timed)
+    step_ms = reduce_max(fwd_ms + bwd_ms, world)
+    if rank != 0:
+        return
+    peaks, peak_kind = load_peaks()
+    total = fwd_flops * (3.5 if train else 1.0)
+    value = world * total / (step_ms / 1e3) / 1e12
+    line = {
+        "metric": ("one-shot chunk-causal attn fwd+bwd TFLOP/s" if train else
+                   "one-shot chunk-causal attn fwd TFLOP/s"),
+        "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded N(0,1) bf16 Q/K/V/dO)",
+        "config": {"workload": w.name, "batch": w.batch, "heads": w.heads,
+                   "head_dim": w.head_dim, "tokens": w.num_tokens,
+                   "frames_per_chunk": w.frames_per_chunk,
+                   "window_chunks": w.window_chunks, "mode": args.mode},
+        "fwd_ms": fwd_ms, "fwd_tflops": fwd_flops / (fwd_ms / 1e3) / 1e12,
+        "fwd_frac_of_burst_peak": fwd_flops / (fwd_ms / 1e3) / 1e12 /
+                                  peaks["bf16_tflops"],
+    }
+    if train:
+        line["bwd_ms"] = bwd_ms
+        line["bwd_tflops"] = 2.5 * fwd_flops / (bwd_ms / 1e3) / 1e12
+        line["bwd_frac_of_burst_peak"] = line["bwd_tflops"] / peaks["bf16_tflops"]
+    print(json.dumps(line), flush=True)
+
+
 def run_e2e(args, w, chunks, att, dev, step_flops, world):
     """The same metric through the public API from pinned host buffers: every
     step copies each chunk's Q/K/V host->device (a side stream, overlapped
@@ -477,6 +544,11 @@ def main(argv=None):
     ap.add_argument("--chunks", type=int, default=0,
                     help="stream only the first N chunks (small profiling "
                          "cases); 0 = the whole workload")
+    ap.add_argument("--mode", default="stream",
+                    choices=["stream", "oneshot", "train"],
+                    help="stream: the streaming metric (default); oneshot / "
+                         "train: the whole sequence at once, forward / "
+                         "forward + backward (extra measurements)")
     ap.add_argument("--skip-e2e", action="store_true",
                     help="omit the end-to-end leg (profiling cases)")
     args = ap.parse_args(argv)
@@ -496,7 +568,10 @@ def main(argv=None):
         torch.cuda.set_device(local_rank)
         dist.init_process_group("nccl")
     try:
-        run_gpu(args, rank, world, local_rank)
+        if args.mode == "stream":
+            run_gpu(args, rank, world, local_rank)
+        else:
+            run_oneshot(args, rank, world, local_rank)
     finally:
         if world > 1:
             import torch.distributed as dist

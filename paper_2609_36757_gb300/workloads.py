@@ -88,9 +88,15 @@ PAPER_TILES_32 = Workload("paper-tiles-32x32", 6, 24, 128, 32 * 32, 3, 10,
 PAPER_TILES_64 = Workload("paper-tiles-64x64", 6, 24, 128, 64 * 64, 3, 10,
                           window_chunks=1, seed=6)
 
+# A training clip (Sec. 4.1: 45-frame clips at 1024 x 1024): 12 latent frames
+# (4x temporal, 16x spatial reduction, 2 x 2 patch -> 32 x 32 tokens), chunks
+# of 3 frames, one predecessor visible (Eq. 1), processed in one shot.
+TRAIN_CLIP = Workload("train-1024-clip", 1, 24, 128, 32 * 32, 3, 4,
+                      window_chunks=1, seed=7)
+
 WORKLOADS = {w.name: w for w in
              (TINY, W480P, W720P_PEAKED, W1080P, W1080P_WINDOWED,
-              PAPER_TILES_32, PAPER_TILES_64)}
+              PAPER_TILES_32, PAPER_TILES_64, TRAIN_CLIP)}
 
 
 def chunk_stream(w: Workload) -> Iterator[Tuple[int, torch.Tensor, torch.Tensor,
