@@ -38,7 +38,9 @@ using namespace sm100;
 constexpr int kT = 128;           // tile rows (TMEM lanes) and tile columns
 constexpr int kBox = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr int kStages = 2;        // streamed-operand ring depth
-constexpr int kThreads = 192;     // 4 compute warps, producer, MMA issuer
+constexpr int kThreads = 320;     // 8 compute warps, producer, MMA issuer
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
@@ -135,21 +137,21 @@ __device__ __forceinline__ void query_sees(const BwdParams& p, int row, int& lo,
   hi = min((c + 1) * p.chunk_tokens, p.seq_tokens);
 }
 
-// Common CTA prologue: TMEM (warp 5) and barriers (thread 128).
+// Common CTA prologue: TMEM (MMA warp) and barriers (producer thread).
 __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
   const int warp = threadIdx.x / 32;
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     tmem_alloc(&S->tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  if (threadIdx.x == 128) {
+  if (threadIdx.x == kProducerWarp * 32) {
     mbar_init(&S->fixed_full, 1);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&S->full[s], 1);
       mbar_init(&S->empty[s], 1);
     }
     mbar_init(&S->s_full, 1);
-    mbar_init(&S->p_full, 4 * 32);
+    mbar_init(&S->p_full, 8 * 32);
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -164,7 +166,7 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
 __device__ __forceinline__ void bwd_teardown(uint32_t tmem) {
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x / 32 == 5) {
+  if (threadIdx.x / 32 == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -227,15 +229,17 @@ __device__ __forceinline__ void mma_nt(uint32_t sbase, uint32_t tmem, int c0,
   }
 }
 
-// D (+)= A_tmem (128 x 128, bf16 pairs at column a0) * B, B an MN-major
-// [128 x d] tile at SMEM offset b_off: TMEM column c0.
+// D (+)= A_tmem * B, B an MN-major [128 x d] tile at SMEM offset b_off:
+// TMEM column c0.  A is 128 x 128 bf16 written by the compute warps in two
+// halves of 64 K-columns, each half's 32 packed columns at the start of its
+// own 64-column range: K step kk (16 columns) is at a0 + 64 (kk / 4) + 8 (kk % 4).
 template <int D>
 __device__ __forceinline__ void mma_tn(uint32_t sbase, uint32_t tmem, int c0,
                                        int a0, int b_off, int acc) {
   constexpr uint32_t kIdesc = idesc_bf16_f32(kT, D, 1);
 #pragma unroll
   for (int kk = 0; kk < kT / 16; ++kk)
-    mma_ts(tmem + c0, tmem + a0 + kk * 8,
+    mma_ts(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
            smem_desc_sw128(sbase + b_off + kk * 2048, kBox, 1024), kIdesc,
            (acc | kk) != 0);
 }
@@ -256,6 +260,59 @@ __device__ __forceinline__ void store_row32(uint32_t taddr, float mul,
 #pragma unroll
     for (int v = 0; v < 4; ++v)
       d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+  }
+}
+
+// P and dS for 32 columns [c0, c0 + 32) of a half row: p = 2^(s c2 - lse2),
+// ds = p (dp - D); columns outside [lo, hi) are masked (p = 0).  lse2 and dlt
+// point at this half's 64 per-column values (16-byte aligned).
+__device__ __forceinline__ void p_ds32(const uint32_t (&s)[32],
+                                       const uint32_t (&dp)[32],
+                                       const float* lse2, const float* dlt,
+                                       int c0, int lo, int hi, bool need_mask,
+                                       float c2, uint32_t (&pp)[16],
+                                       uint32_t (&pd)[16]) {
+  float l[32], d[32];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 a = reinterpret_cast<const float4*>(lse2 + c0)[i];
+    const float4 g = reinterpret_cast<const float4*>(dlt + c0)[i];
+    l[4 * i] = a.x, l[4 * i + 1] = a.y, l[4 * i + 2] = a.z, l[4 * i + 3] = a.w;
+    d[4 * i] = g.x, d[4 * i + 1] = g.y, d[4 * i + 2] = g.z, d[4 * i + 3] = g.w;
+  }
+#pragma unroll
+  for (int e = 0; e < 16; ++e) {
+    float pv[2], dv[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int i = 2 * e + u;
+      float x = fmaf(__uint_as_float(s[i]), c2, -l[i]);
+      if (need_mask && (c0 + i < lo || c0 + i >= hi)) x = -INFINITY;
+      pv[u] = ex2(x);
+      dv[u] = pv[u] * (__uint_as_float(dp[i]) - d[i]);
+    }
+    pp[e] = pack_bf16(pv[0], pv[1]);
+    pd[e] = pack_bf16(dv[0], dv[1]);
+  }
+}
+
+// The same with one row value of lse2 and D (dq: the row is a query).
+__device__ __forceinline__ void ds32_row(const uint32_t (&s)[32],
+                                         const uint32_t (&dp)[32], float lse2,
+                                         float dlt, int c0, int lo, int hi,
+                                         bool need_mask, float c2,
+                                         uint32_t (&pd)[16]) {
+#pragma unroll
+  for (int e = 0; e < 16; ++e) {
+    float dv[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int i = 2 * e + u;
+      float x = fmaf(__uint_as_float(s[i]), c2, -lse2);
+      if (need_mask && (c0 + i < lo || c0 + i >= hi)) x = -INFINITY;
+      dv[u] = ex2(x) * (__uint_as_float(dp[i]) - dlt);
+    }
+    pd[e] = pack_bf16(dv[0], dv[1]);
   }
 }
 
@@ -288,14 +345,14 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
   const int n = (q1 - q0 + kT - 1) / kT;
   const uint32_t tmem = bwd_setup(S);
 
-  if (warp == 4) {
+  if (warp == kProducerWarp) {
     if (lane == 0)
       bwd_producer<D, true>(smem, S, &p.k_map, &p.v_map, k0, &p.q_map,
                             &p.do_map, q0, n, h, b,
                             p.lse2 + (int64_t)bh_row(p, b, h) * p.padded,
                             p.delta + (int64_t)bh_row(p, b, h) * p.padded);
     __syncwarp();
-  } else if (warp == 5) {
+  } else if (warp == kMmaWarp) {
     if (lane == 0) {
       const uint32_t sbase = smem_addr(smem);
       bool ok = wait_bar(&S->fixed_full, 0, S);
@@ -318,49 +375,43 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     }
     __syncwarp();
   } else {
-    // Compute warps: thread = key row (TMEM lane) of the tile.
-    const int t = threadIdx.x;  // 0..127
-    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    // Compute warps: warp w owns key rows 32 (w % 4) .. + 31 (its TMEM
+    // lanes) and query columns [64 hf, 64 hf + 64) with hf = w / 4; it writes
+    // its bf16 P^T and dS^T over the first 32 of its own S^T and dP^T
+    // columns, so the two warps of a row never touch each other's columns.
+    const int hf = warp / 4;
+    const int t = (warp % 4) * 32 + lane;  // key row within the tile
+    const uint32_t row_t = tmem + ((uint32_t)((warp % 4) * 32) << 16);
+    const uint32_t cs = 64 * hf, cp = 128 + 64 * hf;
     int vis_lo, vis_hi;
     key_sees(p, k0 + t, vis_lo, vis_hi);
     const float c2 = p.scale_log2;
     bool ok = true;
     for (int j = 0; j < n; ++j) {
-      const int i0 = q0 + j * kT;  // first query of the tile
+      const int i0 = q0 + j * kT + 64 * hf;  // first query of this half
       const int st = j % kStages;
       // the stage's LSE and D slices (the MMA warp frees the stage only after
       // p_full, so they stay valid while this tile is processed)
       if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
       if (!(ok = wait_bar(&S->s_full, j & 1, S))) break;
       tc_fence_after();
-      const float* lse2 = S->lse2[st];
-      const float* dlt = S->dlt[st];
+      const float* lse2 = S->lse2[st] + 64 * hf;
+      const float* dlt = S->dlt[st] + 64 * hf;
       const int lo = vis_lo - i0, hi = vis_hi - i0;
-      const bool need_mask = lo > 0 || hi < kT;
-#pragma unroll 1
-      for (int c = 0; c < 4; ++c) {  // 32 query columns at a time
-        uint32_t s[32], dp[32];
-        tmem_ld32(tmem + lane_off + c * 32, s);
-        tmem_ld32(tmem + lane_off + 128 + c * 32, dp);
-        tmem_wait_ld();
-        uint32_t pp[16], pd[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          float pv[2], dv[2];
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int col = c * 32 + 2 * e + u;
-            float x = fmaf(__uint_as_float(s[2 * e + u]), c2, -lse2[col]);
-            if (need_mask && (col < lo || col >= hi)) x = -INFINITY;
-            pv[u] = ex2(x);
-            dv[u] = pv[u] * (__uint_as_float(dp[2 * e + u]) - dlt[col]);
-          }
-          pp[e] = pack_bf16(pv[0], pv[1]);
-          pd[e] = pack_bf16(dv[0], dv[1]);
-        }
-        tmem_st16(tmem + lane_off + c * 16, pp);        // P^T over S^T
-        tmem_st16(tmem + lane_off + 128 + c * 16, pd);  // dS^T over dP^T
-      }
+      const bool need_mask = lo > 0 || hi < 64;
+      uint32_t s0[32], d0[32], s1[32], d1[32], pp[16], pd[16];
+      tmem_ld32(row_t + cs, s0);
+      tmem_ld32(row_t + cp, d0);
+      tmem_wait_ld();
+      tmem_ld32(row_t + cs + 32, s1);  // in flight while the first 32 run
+      tmem_ld32(row_t + cp + 32, d1);
+      p_ds32(s0, d0, lse2, dlt, 0, lo, hi, need_mask, c2, pp, pd);
+      tmem_st16(row_t + cs, pp);       // P^T over S^T (already read)
+      tmem_st16(row_t + cp, pd);       // dS^T over dP^T
+      tmem_wait_ld();
+      p_ds32(s1, d1, lse2, dlt, 32, lo, hi, need_mask, c2, pp, pd);
+      tmem_st16(row_t + cs + 16, pp);
+      tmem_st16(row_t + cp + 16, pd);
       tmem_wait_st();
       tc_fence_before();
       mbar_arrive(&S->p_full);
@@ -373,10 +424,9 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
                           (int64_t)(in_range ? key : 0) * p.heads * D +
                           (int64_t)h * D;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; ++c) {
-        store_row32(tmem + lane_off + 256 + c * 32, 1.f, p.dv + off + c * 32,
-                    in_range);
-        store_row32(tmem + lane_off + 384 + c * 32, p.scale, p.dk + off + c * 32,
+      for (int c = hf * D / 64; c < (hf + 1) * D / 64; ++c) {
+        store_row32(row_t + 256 + c * 32, 1.f, p.dv + off + c * 32, in_range);
+        store_row32(row_t + 384 + c * 32, p.scale, p.dk + off + c * 32,
                     in_range);
       }
     }
@@ -408,12 +458,12 @@ dq_kernel(const __grid_constant__ BwdParams p) {
   const int n = (kv1 - kv0 + kT - 1) / kT;
   const uint32_t tmem = bwd_setup(S);
 
-  if (warp == 4) {
+  if (warp == kProducerWarp) {
     if (lane == 0)
       bwd_producer<D, false>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map,
                              &p.v_map, kv0, n, h, b, nullptr, nullptr);
     __syncwarp();
-  } else if (warp == 5) {
+  } else if (warp == kMmaWarp) {
     if (lane == 0) {
       const uint32_t sbase = smem_addr(smem);
       bool ok = wait_bar(&S->fixed_full, 0, S);
@@ -435,9 +485,13 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     }
     __syncwarp();
   } else {
-    // Compute warps: thread = query row (TMEM lane).
-    const int t = threadIdx.x;
-    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    // Compute warps: warp w owns query rows 32 (w % 4) .. + 31 and key
+    // columns [64 hf, 64 hf + 64), hf = w / 4; dS goes over the first 32 of
+    // its own dP columns.
+    const int hf = warp / 4;
+    const int t = (warp % 4) * 32 + lane;
+    const uint32_t row_t = tmem + ((uint32_t)((warp % 4) * 32) << 16);
+    const uint32_t cs = 64 * hf, cp = 128 + 64 * hf;
     const int row = q0 + t;
     const bool in_range = row < p.seq_tokens;
     int vis_lo, vis_hi;
@@ -448,33 +502,24 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     const float c2 = p.scale_log2;
     bool ok = true;
     for (int j = 0; j < n; ++j) {
-      const int tok0 = kv0 + j * kT;
+      const int tok0 = kv0 + j * kT + 64 * hf;
       if (!(ok = wait_bar(&S->s_full, j & 1, S))) break;
       tc_fence_after();
       const int lo = vis_lo - tok0;
-      const int hi = min(vis_hi, kv1) - tok0;
-      const bool need_mask = lo > 0 || hi < kT || !in_range;
-#pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        uint32_t s[32], dp[32];
-        tmem_ld32(tmem + lane_off + c * 32, s);
-        tmem_ld32(tmem + lane_off + 128 + c * 32, dp);
-        tmem_wait_ld();
-        uint32_t pd[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          float dv[2];
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int col = c * 32 + 2 * e + u;
-            float x = fmaf(__uint_as_float(s[2 * e + u]), c2, -lse2);
-            if (need_mask && (col < lo || col >= hi || !in_range)) x = -INFINITY;
-            dv[u] = ex2(x) * (__uint_as_float(dp[2 * e + u]) - dlt);
-          }
-          pd[e] = pack_bf16(dv[0], dv[1]);
-        }
-        tmem_st16(tmem + lane_off + 128 + c * 16, pd);  // dS over dP
-      }
+      const int hi = vis_hi - tok0;
+      const bool need_mask = lo > 0 || hi < 64 || !in_range;
+      const int lo_m = in_range ? lo : 64, hi_m = in_range ? hi : 0;
+      uint32_t s0[32], d0[32], s1[32], d1[32], pd[16];
+      tmem_ld32(row_t + cs, s0);
+      tmem_ld32(row_t + cp, d0);
+      tmem_wait_ld();
+      tmem_ld32(row_t + cs + 32, s1);
+      tmem_ld32(row_t + cp + 32, d1);
+      ds32_row(s0, d0, lse2, dlt, 0, lo_m, hi_m, need_mask, c2, pd);
+      tmem_st16(row_t + cp, pd);  // dS over dP (already read)
+      tmem_wait_ld();
+      ds32_row(s1, d1, lse2, dlt, 32, lo_m, hi_m, need_mask, c2, pd);
+      tmem_st16(row_t + cp + 16, pd);
       tmem_wait_st();
       tc_fence_before();
       mbar_arrive(&S->p_full);
@@ -485,8 +530,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
                           (int64_t)(in_range ? row : 0) * p.heads * D +
                           (int64_t)h * D;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; ++c)
-        store_row32(tmem + lane_off + 256 + c * 32, p.scale, p.dq + off + c * 32,
+      for (int c = hf * D / 64; c < (hf + 1) * D / 64; ++c)
+        store_row32(row_t + 256 + c * 32, p.scale, p.dq + off + c * 32,
                     in_range);
     }
   }
