@@ -10,12 +10,13 @@
 // Three kernels, no atomics:
 //   delta_kernel  D_i = <dO_i, O_i> (fp32) into the caller's scratch;
 //   dkdv_kernel   one CTA per 128-key tile: for every query tile that sees it
-//                 S^T = K Q^T and dP^T = V dO^T (SMEM x SMEM -> TMEM), then
-//                 P^T and dS^T in bf16 over them in TMEM, then
-//                 dV += P^T dO and dK += dS^T Q (A from TMEM, B = dO or Q
-//                 read as an MN-major operand);
+//                 S^T = K Q^T and dP^T = V dO^T (SMEM x SMEM -> TMEM); P^T in
+//                 bf16 over S^T while dP^T is computed; dV += P^T dO while
+//                 dS^T is written over dP^T; then dK += dS^T Q (A from TMEM,
+//                 B = dO or Q read as an MN-major operand);
 //   dq_kernel     one CTA per 128-query tile: for every visible key tile
-//                 S = Q K^T, dP = dO V^T, dS, dQ += dS K.
+//                 S = Q K^T and dP = dO V^T; P in registers (then the next
+//                 tile's S is issued), dS over dP, dQ += dS K.
 // Visibility is Eq. 1 with window W per (query row, key): a key of chunk c'
 // is seen by queries of chunks c' .. c' + W, a query of chunk c sees keys of
 // chunks c - W .. c; only tiles inside a CTA's visible range are loaded and
@@ -46,8 +47,8 @@ constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
 struct BwdParams {
   CUtensorMap q_map, k_map, v_map, do_map;  // {d, L, H, B} token-major
-  const float* lse2;   // forward LSE in log2 units [B*H, Lpad] (scratch)
-  const float* delta;  // D [B*H, Lpad] (scratch); padding tokens hold 0
+  const float* lse2;   // -(forward LSE in log2 units) [B*H, Lpad] (scratch)
+  const float* delta;  // -D [B*H, Lpad] (scratch); padding tokens hold 0
   uint16_t* dq;        // bf16 [B, L, H, d]
   uint16_t* dk;
   uint16_t* dv;
@@ -58,10 +59,10 @@ struct BwdParams {
 struct BwdShared {
   uint64_t fixed_full;                 // the CTA's resident operands
   uint64_t full[kStages], empty[kStages];
-  uint64_t s_full, p_full, o_full, drain;
+  uint64_t s_ready, dp_ready, p_ready, ds_ready, o_full, drain;
   uint32_t tmem_base;
   int abort;
-  // dkdv: the streamed query tile's log2 LSE and D, one slice per stage
+  // dkdv: the streamed query tile's -log2 LSE and -D, one slice per stage
   __align__(16) float lse2[kStages][kT];
   __align__(16) float dlt[kStages][kT];
 };
@@ -150,8 +151,10 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
       mbar_init(&S->full[s], 1);
       mbar_init(&S->empty[s], 1);
     }
-    mbar_init(&S->s_full, 1);
-    mbar_init(&S->p_full, 8 * 32);
+    mbar_init(&S->s_ready, 1);
+    mbar_init(&S->dp_ready, 1);
+    mbar_init(&S->p_ready, 8 * 32);
+    mbar_init(&S->ds_ready, 8 * 32);
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -263,56 +266,88 @@ __device__ __forceinline__ void store_row32(uint32_t taddr, float mul,
   }
 }
 
-// P and dS for 32 columns [c0, c0 + 32) of a half row: p = 2^(s c2 - lse2),
-// ds = p (dp - D); columns outside [lo, hi) are masked (p = 0).  lse2 and dlt
-// point at this half's 64 per-column values (16-byte aligned).
-__device__ __forceinline__ void p_ds32(const uint32_t (&s)[32],
-                                       const uint32_t (&dp)[32],
-                                       const float* lse2, const float* dlt,
-                                       int c0, int lo, int hi, bool need_mask,
-                                       float c2, uint32_t (&pp)[16],
-                                       uint32_t (&pd)[16]) {
-  float l[32], d[32];
+__device__ __forceinline__ uint64_t f2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// P = 2^(s c2 - lse2) for 32 columns [c0, c0 + 32) of a half row, packed to
+// bf16 pairs; columns outside [lo, hi) are masked (p = 0).  nl holds
+// -lse2 for each column (16-byte aligned) or, with kRow, nl_row for all.
+template <bool kRow>
+__device__ __forceinline__ void p32(const uint32_t (&s)[32], const float* nl,
+                                    float nl_row, int c0, int lo, int hi,
+                                    bool need_mask, uint64_t c2x2,
+                                    uint32_t (&pp)[16]) {
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const float4 a = reinterpret_cast<const float4*>(lse2 + c0)[i];
-    const float4 g = reinterpret_cast<const float4*>(dlt + c0)[i];
-    l[4 * i] = a.x, l[4 * i + 1] = a.y, l[4 * i + 2] = a.z, l[4 * i + 3] = a.w;
-    d[4 * i] = g.x, d[4 * i + 1] = g.y, d[4 * i + 2] = g.z, d[4 * i + 3] = g.w;
-  }
+  for (int q = 0; q < 8; ++q) {  // four columns at a time
+    float4 a;
+    if (kRow)
+      a = make_float4(nl_row, nl_row, nl_row, nl_row);
+    else
+      a = reinterpret_cast<const float4*>(nl + c0)[q];
+    float x[4];
+    f2_split(f2_fma(f2(__uint_as_float(s[4 * q]), __uint_as_float(s[4 * q + 1])),
+                    c2x2, f2(a.x, a.y)), x[0], x[1]);
+    f2_split(f2_fma(f2(__uint_as_float(s[4 * q + 2]), __uint_as_float(s[4 * q + 3])),
+                    c2x2, f2(a.z, a.w)), x[2], x[3]);
+    if (need_mask) {
 #pragma unroll
-  for (int e = 0; e < 16; ++e) {
-    float pv[2], dv[2];
-#pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const int i = 2 * e + u;
-      float x = fmaf(__uint_as_float(s[i]), c2, -l[i]);
-      if (need_mask && (c0 + i < lo || c0 + i >= hi)) x = -INFINITY;
-      pv[u] = ex2(x);
-      dv[u] = pv[u] * (__uint_as_float(dp[i]) - d[i]);
+      for (int u = 0; u < 4; ++u) {
+        const int col = c0 + 4 * q + u;
+        if (col < lo || col >= hi) x[u] = -INFINITY;
+      }
     }
-    pp[e] = pack_bf16(pv[0], pv[1]);
-    pd[e] = pack_bf16(dv[0], dv[1]);
+    pp[2 * q] = pack_bf16(ex2(x[0]), ex2(x[1]));
+    pp[2 * q + 1] = pack_bf16(ex2(x[2]), ex2(x[3]));
   }
 }
 
-// The same with one row value of lse2 and D (dq: the row is a query).
-__device__ __forceinline__ void ds32_row(const uint32_t (&s)[32],
-                                         const uint32_t (&dp)[32], float lse2,
-                                         float dlt, int c0, int lo, int hi,
-                                         bool need_mask, float c2,
-                                         uint32_t (&pd)[16]) {
+// dS = P (dP - D) for 32 columns: P as 16 bf16 pairs (read back from TMEM),
+// dP fp32; nd holds -D per column or, with kRow, nd_row for all.
+template <bool kRow>
+__device__ __forceinline__ void ds32(const uint32_t (&pb)[16],
+                                     const uint32_t (&dp)[32], const float* nd,
+                                     float nd_row, int c0, uint32_t (&pd)[16]) {
 #pragma unroll
-  for (int e = 0; e < 16; ++e) {
-    float dv[2];
-#pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const int i = 2 * e + u;
-      float x = fmaf(__uint_as_float(s[i]), c2, -lse2);
-      if (need_mask && (c0 + i < lo || c0 + i >= hi)) x = -INFINITY;
-      dv[u] = ex2(x) * (__uint_as_float(dp[i]) - dlt);
-    }
-    pd[e] = pack_bf16(dv[0], dv[1]);
+  for (int q = 0; q < 8; ++q) {
+    float4 g;
+    if (kRow)
+      g = make_float4(nd_row, nd_row, nd_row, nd_row);
+    else
+      g = reinterpret_cast<const float4*>(nd + c0)[q];
+    float r[4];
+    f2_split(f2_mul(f2(bf16_lo(pb[2 * q]), bf16_hi(pb[2 * q])),
+                    f2_add(f2(__uint_as_float(dp[4 * q]),
+                              __uint_as_float(dp[4 * q + 1])), f2(g.x, g.y))),
+             r[0], r[1]);
+    f2_split(f2_mul(f2(bf16_lo(pb[2 * q + 1]), bf16_hi(pb[2 * q + 1])),
+                    f2_add(f2(__uint_as_float(dp[4 * q + 2]),
+                              __uint_as_float(dp[4 * q + 3])), f2(g.z, g.w))),
+             r[2], r[3]);
+    pd[2 * q] = pack_bf16(r[0], r[1]);
+    pd[2 * q + 1] = pack_bf16(r[2], r[3]);
   }
 }
 
@@ -361,11 +396,14 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
         if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
         tc_fence_after();
         mma_nt<D>(sbase, tmem, 0, 0, st, 0);    // S^T = K Q^T
-        mma_nt<D>(sbase, tmem, 128, 1, st, 1);  // dP^T = V dO^T
-        mma_commit(&S->s_full);
-        if (!(ok = wait_bar(&S->p_full, j & 1, S))) break;
+        mma_commit(&S->s_ready);
+        mma_nt<D>(sbase, tmem, 128, 1, st, 1);  // dP^T = V dO^T (overlaps P)
+        mma_commit(&S->dp_ready);
+        if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
+        if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
+        tc_fence_after();
         mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
         mma_commit(&S->empty[st]);
       }
@@ -385,36 +423,49 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     const uint32_t cs = 64 * hf, cp = 128 + 64 * hf;
     int vis_lo, vis_hi;
     key_sees(p, k0 + t, vis_lo, vis_hi);
-    const float c2 = p.scale_log2;
+    const uint64_t c2x2 = f2(p.scale_log2, p.scale_log2);
     bool ok = true;
     for (int j = 0; j < n; ++j) {
       const int i0 = q0 + j * kT + 64 * hf;  // first query of this half
       const int st = j % kStages;
       // the stage's LSE and D slices (the MMA warp frees the stage only after
-      // p_full, so they stay valid while this tile is processed)
+      // ds_ready, so they stay valid while this tile is processed)
       if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
-      if (!(ok = wait_bar(&S->s_full, j & 1, S))) break;
+      if (!(ok = wait_bar(&S->s_ready, j & 1, S))) break;
       tc_fence_after();
-      const float* lse2 = S->lse2[st] + 64 * hf;
-      const float* dlt = S->dlt[st] + 64 * hf;
+      const float* nl = S->lse2[st] + 64 * hf;  // -log2 LSE per column
+      const float* nd = S->dlt[st] + 64 * hf;   // -D per column
       const int lo = vis_lo - i0, hi = vis_hi - i0;
       const bool need_mask = lo > 0 || hi < 64;
-      uint32_t s0[32], d0[32], s1[32], d1[32], pp[16], pd[16];
-      tmem_ld32(row_t + cs, s0);
-      tmem_ld32(row_t + cp, d0);
+      uint32_t x0[32], x1[32], pk[16];
+      // phase 1 (overlaps the dP^T MMAs): P^T over the first half of S^T
+      tmem_ld32(row_t + cs, x0);
+      tmem_ld32(row_t + cs + 32, x1);
       tmem_wait_ld();
-      tmem_ld32(row_t + cs + 32, s1);  // in flight while the first 32 run
-      tmem_ld32(row_t + cp + 32, d1);
-      p_ds32(s0, d0, lse2, dlt, 0, lo, hi, need_mask, c2, pp, pd);
-      tmem_st16(row_t + cs, pp);       // P^T over S^T (already read)
-      tmem_st16(row_t + cp, pd);       // dS^T over dP^T
-      tmem_wait_ld();
-      p_ds32(s1, d1, lse2, dlt, 32, lo, hi, need_mask, c2, pp, pd);
-      tmem_st16(row_t + cs + 16, pp);
-      tmem_st16(row_t + cp + 16, pd);
+      p32<false>(x0, nl, 0.f, 0, lo, hi, need_mask, c2x2, pk);
+      tmem_st16(row_t + cs, pk);
+      p32<false>(x1, nl, 0.f, 32, lo, hi, need_mask, c2x2, pk);
+      tmem_st16(row_t + cs + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&S->p_full);
+      mbar_arrive(&S->p_ready);
+      // phase 2 (overlaps the dV MMAs): dS^T over the first half of dP^T,
+      // with P^T read back (bf16) from TMEM
+      if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
+      tc_fence_after();
+      uint32_t pb0[16], pb1[16];
+      tmem_ld16(row_t + cs, pb0);
+      tmem_ld16(row_t + cs + 16, pb1);
+      tmem_ld32(row_t + cp, x0);
+      tmem_ld32(row_t + cp + 32, x1);
+      tmem_wait_ld();
+      ds32<false>(pb0, x0, nd, 0.f, 0, pk);
+      tmem_st16(row_t + cp, pk);
+      ds32<false>(pb1, x1, nd, 0.f, 32, pk);
+      tmem_st16(row_t + cp + 16, pk);
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&S->ds_ready);
     }
     if (ok && wait_bar(&S->o_full, 0, S)) {
       tc_fence_after();
@@ -466,18 +517,33 @@ dq_kernel(const __grid_constant__ BwdParams p) {
   } else if (warp == kMmaWarp) {
     if (lane == 0) {
       const uint32_t sbase = smem_addr(smem);
-      bool ok = wait_bar(&S->fixed_full, 0, S);
-      for (int j = 0; ok && j < n; ++j) {
-        const int st = j % kStages;
-        if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
+      // S of the next tile is issued as soon as P of this one is in
+      // registers, so it overlaps the dS computation.
+      bool ok = wait_bar(&S->fixed_full, 0, S) && wait_bar(&S->full[0], 0, S);
+      if (ok) {
         tc_fence_after();
-        mma_nt<D>(sbase, tmem, 0, 0, st, 0);    // S = Q K^T
-        mma_nt<D>(sbase, tmem, 128, 1, st, 1);  // dP = dO V^T
-        mma_commit(&S->s_full);
-        if (!(ok = wait_bar(&S->p_full, j & 1, S))) break;
+        mma_nt<D>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
+        mma_commit(&S->s_ready);
+        mma_nt<D>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
+        mma_commit(&S->dp_ready);
+      }
+      for (int j = 0; ok && j < n; ++j) {
+        const int st = j % kStages, stn = (j + 1) % kStages;
+        if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
+        if (j + 1 < n) {
+          if (!(ok = wait_bar(&S->full[stn], ((j + 1) / kStages) & 1, S))) break;
+          tc_fence_after();
+          mma_nt<D>(sbase, tmem, 0, 0, stn, 0);  // S_{j+1}
+          mma_commit(&S->s_ready);
+        }
+        if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 256, 128, L::ring(st, 0, 0), j > 0);  // dQ
         mma_commit(&S->empty[st]);
+        if (j + 1 < n) {
+          mma_nt<D>(sbase, tmem, 128, 1, stn, 1);  // dP_{j+1}
+          mma_commit(&S->dp_ready);
+        }
       }
       if (ok) mma_commit(&S->o_full);
       mma_commit(&S->drain);
@@ -497,32 +563,41 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     int vis_lo, vis_hi;
     query_sees(p, row, vis_lo, vis_hi);
     const int64_t rl = (int64_t)bh_row(p, b, h) * p.padded + row;
-    const float lse2 = p.lse2[rl];  // the padded rows hold 0
-    const float dlt = p.delta[rl];
-    const float c2 = p.scale_log2;
+    const float nl_row = p.lse2[rl];  // -log2 LSE (padded rows hold 0)
+    const float nd_row = p.delta[rl];  // -D
+    const uint64_t c2x2 = f2(p.scale_log2, p.scale_log2);
     bool ok = true;
     for (int j = 0; j < n; ++j) {
       const int tok0 = kv0 + j * kT + 64 * hf;
-      if (!(ok = wait_bar(&S->s_full, j & 1, S))) break;
+      if (!(ok = wait_bar(&S->s_ready, j & 1, S))) break;
       tc_fence_after();
       const int lo = vis_lo - tok0;
       const int hi = vis_hi - tok0;
       const bool need_mask = lo > 0 || hi < 64 || !in_range;
       const int lo_m = in_range ? lo : 64, hi_m = in_range ? hi : 0;
-      uint32_t s0[32], d0[32], s1[32], d1[32], pd[16];
-      tmem_ld32(row_t + cs, s0);
-      tmem_ld32(row_t + cp, d0);
+      uint32_t x0[32], x1[32], pb0[16], pb1[16], pk[16];
+      // phase 1 (overlaps the dP MMAs): P (bf16 pairs) in registers; S is
+      // then free for the next tile
+      tmem_ld32(row_t + cs, x0);
+      tmem_ld32(row_t + cs + 32, x1);
       tmem_wait_ld();
-      tmem_ld32(row_t + cs + 32, s1);
-      tmem_ld32(row_t + cp + 32, d1);
-      ds32_row(s0, d0, lse2, dlt, 0, lo_m, hi_m, need_mask, c2, pd);
-      tmem_st16(row_t + cp, pd);  // dS over dP (already read)
+      p32<true>(x0, nullptr, nl_row, 0, lo_m, hi_m, need_mask, c2x2, pb0);
+      p32<true>(x1, nullptr, nl_row, 32, lo_m, hi_m, need_mask, c2x2, pb1);
+      tc_fence_before();
+      mbar_arrive(&S->p_ready);
+      // phase 2 (overlaps the next tile's S MMAs): dS over the dP columns
+      if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
+      tc_fence_after();
+      tmem_ld32(row_t + cp, x0);
+      tmem_ld32(row_t + cp + 32, x1);
       tmem_wait_ld();
-      ds32_row(s1, d1, lse2, dlt, 32, lo_m, hi_m, need_mask, c2, pd);
-      tmem_st16(row_t + cp + 16, pd);
+      ds32<true>(pb0, x0, nullptr, nd_row, 0, pk);
+      tmem_st16(row_t + cp, pk);
+      ds32<true>(pb1, x1, nullptr, nd_row, 32, pk);
+      tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&S->p_full);
+      mbar_arrive(&S->ds_ready);
     }
     if (ok && wait_bar(&S->o_full, 0, S)) {
       tc_fence_after();
@@ -538,10 +613,11 @@ dq_kernel(const __grid_constant__ BwdParams p) {
   bwd_teardown(tmem);
 }
 
-// Scratch rows for the backward: D_i = <dO_i, O_i> over the head dim and
-// the forward LSE in log2 units, each [B*H, Lpad] with Lpad = L rounded up to
-// 128 and zeros in the padding (so every 128-token slice is aligned and in
-// bounds).  One warp per (b, token, head) row of O.
+// Scratch rows for the backward: -D_i = -<dO_i, O_i> over the head dim and
+// minus the forward LSE in log2 units (negated so that both enter packed
+// FMAs as addends), each [B*H, Lpad] with Lpad = L rounded up to 128 and
+// zeros in the padding (so every 128-token slice is aligned and in bounds).
+// One warp per (b, token, head) row of O.
 template <int D>
 __global__ void __launch_bounds__(256)
 delta_kernel(const uint16_t* o, const uint16_t* dO, const float* lse,
@@ -567,8 +643,8 @@ delta_kernel(const uint16_t* o, const uint16_t* dO, const float* lse,
       const int64_t h = r % heads, bt = r / heads;
       const int64_t tok = bt % seq, b = bt / seq;
       const int64_t i = (b * heads + h) * padded + tok;
-      delta[i] = acc;
-      lse2[i] = lse[(b * heads + h) * seq + tok] * 1.4426950408889634f;
+      delta[i] = -acc;
+      lse2[i] = -lse[(b * heads + h) * seq + tok] * 1.4426950408889634f;
     }
   }
   // padding tokens
