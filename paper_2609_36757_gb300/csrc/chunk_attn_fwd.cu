@@ -276,28 +276,35 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   const int n = w.n;
   const bool two = w.nqt == 2;
 
+  // One thread issues every MMA and a tcgen05.mma takes it ~55 clk to issue
+  // against 64 clk of tensor work (M128 N128 K16), so the issue loop carries
+  // no descriptor arithmetic: the descriptor words are formed once here and
+  // each MMA only adds a constant offset (16-byte units) to the low word.
+  const uint32_t hi = desc_hi_sw128(1024);
+  const uint32_t q_lo = desc_lo(sbase + L::q(0, 0), 16);
+  const uint32_t k_lo = desc_lo(sbase + L::k(0, 0), 16);
+  const uint32_t v_lo = desc_lo(sbase + L::v(0, 0), kBox);
+  constexpr uint32_t kStage16 = (uint32_t)(L::kNB * kBox) >> 4;
   // S_t = Q_t K^T: both operands K-major, 128-byte swizzle; a K step of 16
   // elements is 32 bytes inside a 64-column box.
   auto qk = [&](int t, int st) {
+    const uint32_t a0 = q_lo + (uint32_t)(L::q(t, 0) >> 4);
+    const uint32_t b0 = k_lo + (uint32_t)st * kStage16;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
-      const uint32_t off = (ks / 4) * kBox + (ks % 4) * 32;
-      const uint64_t a = smem_desc_sw128(sbase + L::q(t, 0) + off, 16, 1024);
-      const uint64_t bdesc = smem_desc_sw128(sbase + L::k(st, 0) + off, 16, 1024);
-      mma_ss(tmem + t * 128, a, bdesc, kIdescQK, ks > 0);
+      const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
+      mma_ss_w(tmem + t * 128, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
     }
   };
   // O_t += P_t V: P_t from TMEM (8 columns per 16 keys), V MN-major (d
   // contiguous): 16 keys are two 8-row groups (2048 bytes), the two 64-column
   // halves of d are one box apart.
   auto pv = [&](int t, int st, int acc) {
+    const uint32_t b0 = v_lo + (uint32_t)st * kStage16;
 #pragma unroll
-    for (int kk = 0; kk < kBN / 16; ++kk) {
-      const uint64_t bdesc =
-          smem_desc_sw128(sbase + L::v(st, 0) + kk * 2048, kBox, 1024);
-      mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8, bdesc, kIdescPV,
-             (acc | kk) != 0);
-    }
+    for (int kk = 0; kk < kBN / 16; ++kk)
+      mma_ts_w(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
+               b0 + (uint32_t)(kk * 2048 >> 4), hi, kIdescPV, (acc | kk) != 0);
   };
 
   // Test hook: o_full receives no arrival before the end of the stream, so

@@ -207,6 +207,19 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr,
   return d;
 }
 
+// The same descriptor as two 32-bit words, for issue loops that precompute
+// it: the low word holds the start address and the leading byte offset, the
+// high word the stride byte offset, version and swizzle.  Moving the start
+// address within shared memory changes only the low word (the 14-bit field
+// cannot carry: shared addresses are below 256 KB).
+__host__ __device__ constexpr uint32_t desc_lo(uint32_t saddr,
+                                               uint32_t lbo_bytes) {
+  return ((saddr >> 4) & 0x3FFFu) | (((lbo_bytes >> 4) & 0x3FFFu) << 16);
+}
+__host__ __device__ constexpr uint32_t desc_hi_sw128(uint32_t sbo_bytes) {
+  return ((sbo_bytes >> 4) & 0x3FFFu) | (1u << 14) | (2u << 29);
+}
+
 // Instruction descriptor for kind::f16 with bf16 A/B and f32 accumulation:
 // D format bits 4-5 (1 = f32), A format bits 7-9 and B format bits 10-12
 // (1 = bf16), A/B major bits 15/16 (0 = K-major, 1 = MN-major),
@@ -240,6 +253,33 @@ __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem,
       "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(
           d_tmem),
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// mma_ss / mma_ts with the descriptors given as (low, high) words.
+__device__ __forceinline__ void mma_ss_w(uint32_t d_tmem, uint32_t a_lo,
+                                         uint32_t b_lo, uint32_t hi,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 da, {%1, %3};\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n\t}" ::"r"(
+          d_tmem),
+      "r"(a_lo), "r"(b_lo), "r"(hi), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_ts_w(uint32_t d_tmem, uint32_t a_tmem,
+                                         uint32_t b_lo, uint32_t hi,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 db;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %5, p;\n\t}" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(accumulate), "r"(idesc)
       : "memory");
 }
 
