@@ -529,7 +529,11 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     }
     tmem_wait_st();
     tc_fence_before();
-    mbar_arrive(&S->p_full[t]);
+    // One arrival per warp (lane 0, after the warp's stores are complete):
+    // the barrier word sits in shared memory, which queued QK^T MMAs keep
+    // busy, so 32 arrivals per warp would each wait their turn.
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&S->p_full[t]);
   }
   if (!ok || !wait_bar(&S->o_full, 0, S, p.status)) return;
   tc_fence_after();
@@ -671,7 +675,7 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     }
     for (int t = 0; t < kQTiles; ++t) {
       mbar_init(&S->s_full[t], 1);
-      mbar_init(&S->p_full[t], 4 * 32);
+      mbar_init(&S->p_full[t], 4);
     }
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
