@@ -153,8 +153,12 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
     }
     mbar_init(&S->s_ready, 1);
     mbar_init(&S->dp_ready, 1);
-    mbar_init(&S->p_ready, 8 * 32);
-    mbar_init(&S->ds_ready, 8 * 32);
+    // One arrival per compute warp (lane 0, after the warp's TMEM accesses
+    // are complete): the barrier words sit in shared memory, which queued
+    // SMEM x SMEM MMAs keep saturated, so per-thread arrivals would each
+    // wait their turn.
+    mbar_init(&S->p_ready, 8);
+    mbar_init(&S->ds_ready, 8);
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -216,19 +220,24 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
     drain_wait(&S->full[i % kStages], (i / kStages) & 1);
 }
 
+// One thread issues every MMA, and a tcgen05.mma takes it about as long to
+// issue as the tensor pipe takes to run it, so the issue loops carry no
+// descriptor arithmetic: each tile's descriptor low word is formed once per
+// call and the K steps add constant offsets (16-byte units) to it.
+
 // D_t = A_fixed * B_ring^T over the head dim (both K-major): TMEM col c0.
 template <int D>
 __device__ __forceinline__ void mma_nt(uint32_t sbase, uint32_t tmem, int c0,
                                        int fixed_which, int st, int ring_which) {
   using L = BwdLayout<D>;
   constexpr uint32_t kIdesc = idesc_bf16_f32(kT, kT, 0);
+  const uint32_t hi = desc_hi_sw128(1024);
+  const uint32_t a_lo = desc_lo(sbase + L::fixed(fixed_which, 0), 16);
+  const uint32_t b_lo = desc_lo(sbase + L::ring(st, ring_which, 0), 16);
 #pragma unroll
   for (int ks = 0; ks < D / 16; ++ks) {
-    const uint32_t off = (ks / 4) * kBox + (ks % 4) * 32;
-    mma_ss(tmem + c0,
-           smem_desc_sw128(sbase + L::fixed(fixed_which, 0) + off, 16, 1024),
-           smem_desc_sw128(sbase + L::ring(st, ring_which, 0) + off, 16, 1024),
-           kIdesc, ks > 0);
+    const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
+    mma_ss_w(tmem + c0, a_lo + off, b_lo + off, hi, kIdesc, ks > 0);
   }
 }
 
@@ -240,11 +249,12 @@ template <int D>
 __device__ __forceinline__ void mma_tn(uint32_t sbase, uint32_t tmem, int c0,
                                        int a0, int b_off, int acc) {
   constexpr uint32_t kIdesc = idesc_bf16_f32(kT, D, 1);
+  const uint32_t hi = desc_hi_sw128(1024);
+  const uint32_t b_lo = desc_lo(sbase + b_off, kBox);
 #pragma unroll
   for (int kk = 0; kk < kT / 16; ++kk)
-    mma_ts(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
-           smem_desc_sw128(sbase + b_off + kk * 2048, kBox, 1024), kIdesc,
-           (acc | kk) != 0);
+    mma_ts_w(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
+             b_lo + (uint32_t)(kk * 2048 >> 4), hi, kIdesc, (acc | kk) != 0);
 }
 
 // Write 32 fp32 accumulator columns (scaled) of a TMEM row as bf16.
@@ -448,7 +458,8 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       tmem_st16(row_t + cs + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&S->p_ready);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S->p_ready);
       // phase 2 (overlaps the dV MMAs): dS^T over the first half of dP^T,
       // with P^T read back (bf16) from TMEM
       if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
@@ -465,7 +476,8 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&S->ds_ready);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S->ds_ready);
     }
     if (ok && wait_bar(&S->o_full, 0, S)) {
       tc_fence_after();
@@ -584,7 +596,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       p32<true>(x0, nullptr, nl_row, 0, lo_m, hi_m, need_mask, c2x2, pb0);
       p32<true>(x1, nullptr, nl_row, 32, lo_m, hi_m, need_mask, c2x2, pb1);
       tc_fence_before();
-      mbar_arrive(&S->p_ready);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S->p_ready);
       // phase 2 (overlaps the next tile's S MMAs): dS over the dP columns
       if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
       tc_fence_after();
@@ -597,7 +610,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&S->ds_ready);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S->ds_ready);
     }
     if (ok && wait_bar(&S->o_full, 0, S)) {
       tc_fence_after();
