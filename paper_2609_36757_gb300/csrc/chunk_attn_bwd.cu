@@ -11,9 +11,10 @@
 //   delta_kernel  D_i = <dO_i, O_i> (fp32) into the caller's scratch;
 //   dkdv_kernel   one CTA per 128-key tile: for every query tile that sees it
 //                 S^T = K Q^T and dP^T = V dO^T (SMEM x SMEM -> TMEM); P^T in
-//                 bf16 over S^T while dP^T is computed; dV += P^T dO while
-//                 dS^T is written over dP^T; then dK += dS^T Q (A from TMEM,
-//                 B = dO or Q read as an MN-major operand);
+//                 bf16 over S^T (and in registers); dV += P^T dO, then the
+//                 next tile's S^T, while dS^T is written over dP^T; then
+//                 dK += dS^T Q (A from TMEM, B = dO or Q read as an MN-major
+//                 operand) and the next tile's dP^T;
 //   dq_kernel     one CTA per 128-query tile: for every visible key tile
 //                 S = Q K^T and dP = dO V^T; P in registers (then the next
 //                 tile's S is issued), dS over dP, dQ += dS K.
@@ -400,22 +401,38 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
   } else if (warp == kMmaWarp) {
     if (lane == 0) {
       const uint32_t sbase = smem_addr(smem);
-      bool ok = wait_bar(&S->fixed_full, 0, S);
-      for (int j = 0; ok && j < n; ++j) {
-        const int st = j % kStages;
-        if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
+      // The next tile's S^T is issued right after this tile's dV (it
+      // overwrites P^T, which dV has read: the pipe runs in issue order and
+      // the compute warps keep P^T in registers), and the next dP^T right
+      // after dK (over dS^T), so the compute warps start the next tile's P
+      // as soon as they finish this tile's dS.
+      bool ok = wait_bar(&S->fixed_full, 0, S) && wait_bar(&S->full[0], 0, S);
+      if (ok) {
         tc_fence_after();
-        mma_nt<D>(sbase, tmem, 0, 0, st, 0);    // S^T = K Q^T
+        mma_nt<D>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
         mma_commit(&S->s_ready);
-        mma_nt<D>(sbase, tmem, 128, 1, st, 1);  // dP^T = V dO^T (overlaps P)
+        mma_nt<D>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
         mma_commit(&S->dp_ready);
+      }
+      for (int j = 0; ok && j < n; ++j) {
+        const int st = j % kStages, stn = (j + 1) % kStages;
         if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
+        if (j + 1 < n) {
+          if (!(ok = wait_bar(&S->full[stn], ((j + 1) / kStages) & 1, S))) break;
+          tc_fence_after();
+          mma_nt<D>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
+          mma_commit(&S->s_ready);
+        }
         if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
         mma_commit(&S->empty[st]);
+        if (j + 1 < n) {
+          mma_nt<D>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
+          mma_commit(&S->dp_ready);
+        }
       }
       if (ok) mma_commit(&S->o_full);
       mma_commit(&S->drain);
@@ -447,26 +464,25 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       const float* nd = S->dlt[st] + 64 * hf;   // -D per column
       const int lo = vis_lo - i0, hi = vis_hi - i0;
       const bool need_mask = lo > 0 || hi < 64;
-      uint32_t x0[32], x1[32], pk[16];
-      // phase 1 (overlaps the dP^T MMAs): P^T over the first half of S^T
+      uint32_t x0[32], x1[32], pb0[16], pb1[16], pk[16];
+      // phase 1: P^T over the first half of S^T (for the dV MMA) and in
+      // registers (for dS: the next tile's S^T may overwrite it in TMEM as
+      // soon as dV has run)
       tmem_ld32(row_t + cs, x0);
       tmem_ld32(row_t + cs + 32, x1);
       tmem_wait_ld();
-      p32<false>(x0, nl, 0.f, 0, lo, hi, need_mask, c2x2, pk);
-      tmem_st16(row_t + cs, pk);
-      p32<false>(x1, nl, 0.f, 32, lo, hi, need_mask, c2x2, pk);
-      tmem_st16(row_t + cs + 16, pk);
+      p32<false>(x0, nl, 0.f, 0, lo, hi, need_mask, c2x2, pb0);
+      tmem_st16(row_t + cs, pb0);
+      p32<false>(x1, nl, 0.f, 32, lo, hi, need_mask, c2x2, pb1);
+      tmem_st16(row_t + cs + 16, pb1);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->p_ready);
-      // phase 2 (overlaps the dV MMAs): dS^T over the first half of dP^T,
-      // with P^T read back (bf16) from TMEM
+      // phase 2 (overlaps the dV and next S^T MMAs): dS^T over the first
+      // half of dP^T
       if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
       tc_fence_after();
-      uint32_t pb0[16], pb1[16];
-      tmem_ld16(row_t + cs, pb0);
-      tmem_ld16(row_t + cs + 16, pb1);
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
       tmem_wait_ld();
