@@ -304,20 +304,18 @@ __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
 // P = 2^(s c2 - lse2) for 32 columns [c0, c0 + 32) of a half row, packed to
-// bf16 pairs; columns outside [lo, hi) are masked (p = 0).  nl holds
-// -lse2 for each column (16-byte aligned) or, with kRow, nl_row for all.
-template <bool kRow>
-__device__ __forceinline__ void p32(const uint32_t (&s)[32], const float* nl,
-                                    float nl_row, int c0, int lo, int hi,
-                                    bool need_mask, uint64_t c2x2,
+// bf16 pairs; columns outside [lo, hi) are masked (p = 0).  nl holds -lse2
+// for the 32 columns, in registers: the dK/dV kernel reads its per-column
+// values from shared memory ahead of use, because the SMEM x SMEM MMAs that
+// run meanwhile take all of the shared-memory bandwidth and each read waits
+// behind them.
+__device__ __forceinline__ void p32(const uint32_t (&s)[32],
+                                    const float4 (&nl)[8], int c0, int lo,
+                                    int hi, bool need_mask, uint64_t c2x2,
                                     uint32_t (&pp)[16]) {
 #pragma unroll
   for (int q = 0; q < 8; ++q) {  // four columns at a time
-    float4 a;
-    if (kRow)
-      a = make_float4(nl_row, nl_row, nl_row, nl_row);
-    else
-      a = reinterpret_cast<const float4*>(nl + c0)[q];
+    const float4 a = nl[q];
     float x[4];
     f2_split(f2_fma(f2(__uint_as_float(s[4 * q]), __uint_as_float(s[4 * q + 1])),
                     c2x2, f2(a.x, a.y)), x[0], x[1]);
@@ -335,19 +333,14 @@ __device__ __forceinline__ void p32(const uint32_t (&s)[32], const float* nl,
   }
 }
 
-// dS = P (dP - D) for 32 columns: P as 16 bf16 pairs (read back from TMEM),
-// dP fp32; nd holds -D per column or, with kRow, nd_row for all.
-template <bool kRow>
+// dS = P (dP - D) for 32 columns: P as 16 bf16 pairs, dP fp32, nd holds -D
+// for the 32 columns in registers.
 __device__ __forceinline__ void ds32(const uint32_t (&pb)[16],
-                                     const uint32_t (&dp)[32], const float* nd,
-                                     float nd_row, int c0, uint32_t (&pd)[16]) {
+                                     const uint32_t (&dp)[32],
+                                     const float4 (&nd)[8], uint32_t (&pd)[16]) {
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
-    float4 g;
-    if (kRow)
-      g = make_float4(nd_row, nd_row, nd_row, nd_row);
-    else
-      g = reinterpret_cast<const float4*>(nd + c0)[q];
+    const float4 g = nd[q];
     float r[4];
     f2_split(f2_mul(f2(bf16_lo(pb[2 * q]), bf16_hi(pb[2 * q])),
                     f2_add(f2(__uint_as_float(dp[4 * q]),
@@ -458,10 +451,14 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       // the stage's LSE and D slices (the MMA warp frees the stage only after
       // ds_ready, so they stay valid while this tile is processed)
       if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
-      if (!(ok = wait_bar(&S->s_ready, j & 1, S))) break;
-      tc_fence_after();
       const float* nl = S->lse2[st] + 64 * hf;  // -log2 LSE per column
       const float* nd = S->dlt[st] + 64 * hf;   // -D per column
+      // the first half's LSE values land while S^T is computed
+      float4 la[8], lb[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) la[q] = reinterpret_cast<const float4*>(nl)[q];
+      if (!(ok = wait_bar(&S->s_ready, j & 1, S))) break;
+      tc_fence_after();
       const int lo = vis_lo - i0, hi = vis_hi - i0;
       const bool need_mask = lo > 0 || hi < 64;
       uint32_t x0[32], x1[32], pb0[16], pb1[16], pk[16];
@@ -470,25 +467,33 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       // soon as dV has run)
       tmem_ld32(row_t + cs, x0);
       tmem_ld32(row_t + cs + 32, x1);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        lb[q] = reinterpret_cast<const float4*>(nl + 32)[q];
       tmem_wait_ld();
-      p32<false>(x0, nl, 0.f, 0, lo, hi, need_mask, c2x2, pb0);
+      p32(x0, la, 0, lo, hi, need_mask, c2x2, pb0);
       tmem_st16(row_t + cs, pb0);
-      p32<false>(x1, nl, 0.f, 32, lo, hi, need_mask, c2x2, pb1);
+      p32(x1, lb, 32, lo, hi, need_mask, c2x2, pb1);
       tmem_st16(row_t + cs + 16, pb1);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->p_ready);
       // phase 2 (overlaps the dV and next S^T MMAs): dS^T over the first
-      // half of dP^T
+      // half of dP^T; the D values are read ahead like the LSE values
+#pragma unroll
+      for (int q = 0; q < 8; ++q) la[q] = reinterpret_cast<const float4*>(nd)[q];
       if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
       tc_fence_after();
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        lb[q] = reinterpret_cast<const float4*>(nd + 32)[q];
       tmem_wait_ld();
-      ds32<false>(pb0, x0, nd, 0.f, 0, pk);
+      ds32(pb0, x0, la, pk);
       tmem_st16(row_t + cp, pk);
-      ds32<false>(pb1, x1, nd, 0.f, 32, pk);
+      ds32(pb1, x1, lb, pk);
       tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
@@ -592,7 +597,13 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     query_sees(p, row, vis_lo, vis_hi);
     const int64_t rl = (int64_t)bh_row(p, b, h) * p.padded + row;
     const float nl_row = p.lse2[rl];  // -log2 LSE (padded rows hold 0)
+    float4 nl_v[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) nl_v[q] = make_float4(nl_row, nl_row, nl_row, nl_row);
     const float nd_row = p.delta[rl];  // -D
+    float4 nd_v[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) nd_v[q] = make_float4(nd_row, nd_row, nd_row, nd_row);
     const uint64_t c2x2 = f2(p.scale_log2, p.scale_log2);
     bool ok = true;
     for (int j = 0; j < n; ++j) {
@@ -609,8 +620,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tmem_ld32(row_t + cs, x0);
       tmem_ld32(row_t + cs + 32, x1);
       tmem_wait_ld();
-      p32<true>(x0, nullptr, nl_row, 0, lo_m, hi_m, need_mask, c2x2, pb0);
-      p32<true>(x1, nullptr, nl_row, 32, lo_m, hi_m, need_mask, c2x2, pb1);
+      p32(x0, nl_v, 0, lo_m, hi_m, need_mask, c2x2, pb0);
+      p32(x1, nl_v, 32, lo_m, hi_m, need_mask, c2x2, pb1);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->p_ready);
@@ -620,9 +631,9 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
       tmem_wait_ld();
-      ds32<true>(pb0, x0, nullptr, nd_row, 0, pk);
+      ds32(pb0, x0, nd_v, pk);
       tmem_st16(row_t + cp, pk);
-      ds32<true>(pb1, x1, nullptr, nd_row, 32, pk);
+      ds32(pb1, x1, nd_v, pk);
       tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
