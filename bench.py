@@ -300,7 +300,9 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
     fwd_total_ms = sum(map(sum, fwd_ms))
     attn_tflops = step_flops * args.steps / (fwd_total_ms / 1e3) / 1e12
     app_total_ms = sum(map(sum, app_ms))
-    app_bytes = sum(2 * 2 * w.batch * w.heads * w.frames_in_chunk(c) *
+    # K and V (bf16) read once and written once: read + write bytes, the
+    # same accounting as the measured HBM copy peak
+    app_bytes = sum(2 * 2 * 2 * w.batch * w.heads * w.frames_in_chunk(c) *
                     w.tokens_per_frame * w.head_dim for c in range(w.num_chunks))
     app_gbs = app_bytes * args.steps / (app_total_ms / 1e3) / 1e9
     per_chunk_fwd = [statistics.median(fwd_ms[s][c] for s in range(args.steps))
