@@ -59,7 +59,12 @@ struct BwdParams {
 
 struct BwdShared {
   uint64_t fixed_full;                 // the CTA's resident operands
-  uint64_t full[kStages], empty[kStages];
+  // Two streamed rings with their own barriers, [ring][stage]: ring 0 holds
+  // the tile read last in a step (dq: K, read by dQ; dkdv: Q and the row
+  // vectors, read by dK), ring 1 the other (dq: V, last read by dP; dkdv:
+  // dO, last read by dV), so a ring-1 slot is refilled as soon as its last
+  // reader has run instead of waiting for the end of the step.
+  uint64_t full[2][kStages], empty[2][kStages];
   uint64_t s_ready, dp_ready, p_ready, ds_ready, o_full, drain;
   uint32_t tmem_base;
   int abort;
@@ -148,10 +153,11 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
   }
   if (threadIdx.x == kProducerWarp * 32) {
     mbar_init(&S->fixed_full, 1);
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&S->full[s], 1);
-      mbar_init(&S->empty[s], 1);
-    }
+    for (int r = 0; r < 2; ++r)
+      for (int s = 0; s < kStages; ++s) {
+        mbar_init(&S->full[r][s], 1);
+        mbar_init(&S->empty[r][s], 1);
+      }
     mbar_init(&S->s_ready, 1);
     mbar_init(&S->dp_ready, 1);
     // One arrival per compute warp (lane 0, after the warp's TMEM accesses
@@ -197,28 +203,36 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
     tma_load_4d(f0, smem + L::fixed(0, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
     tma_load_4d(f1, smem + L::fixed(1, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
   }
-  int issued = 0;
+  // Ring 1 first: its slot frees earlier in a step (after dP or dV), so its
+  // next tile loads while the step still runs; ring 0 (after dQ or dK)
+  // follows.
+  int issued[2] = {0, 0};
   for (int j = 0; j < n; ++j) {
     const int st = j % kStages;
-    if (!wait_bar(&S->empty[st], ((j / kStages) & 1) ^ 1, S)) break;
-    mbar_arrive_expect_tx(&S->full[st], 2 * L::kNB * kBox + kVecBytes);
-    for (int bx = 0; bx < L::kNB; ++bx) {
-      tma_load_4d(r0, smem + L::ring(st, 0, bx), &S->full[st], bx * 64,
+    const uint32_t ph = ((j / kStages) & 1) ^ 1;
+    if (!wait_bar(&S->empty[1][st], ph, S)) break;
+    mbar_arrive_expect_tx(&S->full[1][st], L::kNB * kBox);
+    for (int bx = 0; bx < L::kNB; ++bx)
+      tma_load_4d(r1, smem + L::ring(st, 1, bx), &S->full[1][st], bx * 64,
                   t0 + j * kT, h, b);
-      tma_load_4d(r1, smem + L::ring(st, 1, bx), &S->full[st], bx * 64,
+    ++issued[1];
+    if (!wait_bar(&S->empty[0][st], ph, S)) break;
+    mbar_arrive_expect_tx(&S->full[0][st], L::kNB * kBox + kVecBytes);
+    for (int bx = 0; bx < L::kNB; ++bx)
+      tma_load_4d(r0, smem + L::ring(st, 0, bx), &S->full[0][st], bx * 64,
                   t0 + j * kT, h, b);
-    }
     if (kRowVecs) {
       bulk_load(S->lse2[st], vec_lse2 + t0 + j * kT, kT * sizeof(float),
-                &S->full[st]);
+                &S->full[0][st]);
       bulk_load(S->dlt[st], vec_dlt + t0 + j * kT, kT * sizeof(float),
-                &S->full[st]);
+                &S->full[0][st]);
     }
-    ++issued;
+    ++issued[0];
   }
   drain_wait(&S->fixed_full, 0);
-  for (int i = max(0, issued - kStages); i < issued; ++i)
-    drain_wait(&S->full[i % kStages], (i / kStages) & 1);
+  for (int r = 0; r < 2; ++r)
+    for (int i = max(0, issued[r] - kStages); i < issued[r]; ++i)
+      drain_wait(&S->full[r][i % kStages], (i / kStages) & 1);
 }
 
 // One thread issues every MMA, and a tcgen05.mma takes it about as long to
@@ -399,7 +413,8 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       // the compute warps keep P^T in registers), and the next dP^T right
       // after dK (over dS^T), so the compute warps start the next tile's P
       // as soon as they finish this tile's dS.
-      bool ok = wait_bar(&S->fixed_full, 0, S) && wait_bar(&S->full[0], 0, S);
+      bool ok = wait_bar(&S->fixed_full, 0, S) &&
+                wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
       if (ok) {
         tc_fence_after();
         mma_nt<D>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
@@ -409,11 +424,13 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       }
       for (int j = 0; ok && j < n; ++j) {
         const int st = j % kStages, stn = (j + 1) % kStages;
+        const uint32_t phn = ((j + 1) / kStages) & 1;
         if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
+        mma_commit(&S->empty[1][st]);  // dO_j read for the last time
         if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[stn], ((j + 1) / kStages) & 1, S))) break;
+          if (!(ok = wait_bar(&S->full[0][stn], phn, S))) break;
           tc_fence_after();
           mma_nt<D>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
           mma_commit(&S->s_ready);
@@ -421,8 +438,10 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
         if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
-        mma_commit(&S->empty[st]);
+        mma_commit(&S->empty[0][st]);  // Q_j and the row vectors
         if (j + 1 < n) {
+          if (!(ok = wait_bar(&S->full[1][stn], phn, S))) break;
+          tc_fence_after();
           mma_nt<D>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
           mma_commit(&S->dp_ready);
         }
@@ -450,7 +469,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       const int st = j % kStages;
       // the stage's LSE and D slices (the MMA warp frees the stage only after
       // ds_ready, so they stay valid while this tile is processed)
-      if (!(ok = wait_bar(&S->full[st], (j / kStages) & 1, S))) break;
+      if (!(ok = wait_bar(&S->full[0][st], (j / kStages) & 1, S))) break;
       const float* nl = S->lse2[st] + 64 * hf;  // -log2 LSE per column
       const float* nd = S->dlt[st] + 64 * hf;   // -D per column
       // the first half's LSE values land while S^T is computed
@@ -552,19 +571,22 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       const uint32_t sbase = smem_addr(smem);
       // S of the next tile is issued as soon as P of this one is in
       // registers, so it overlaps the dS computation.
-      bool ok = wait_bar(&S->fixed_full, 0, S) && wait_bar(&S->full[0], 0, S);
+      bool ok = wait_bar(&S->fixed_full, 0, S) &&
+                wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
       if (ok) {
         tc_fence_after();
         mma_nt<D>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
         mma_commit(&S->s_ready);
         mma_nt<D>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
         mma_commit(&S->dp_ready);
+        mma_commit(&S->empty[1][0]);           // V_0 read for the last time
       }
       for (int j = 0; ok && j < n; ++j) {
         const int st = j % kStages, stn = (j + 1) % kStages;
+        const uint32_t phn = ((j + 1) / kStages) & 1;
         if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
         if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[stn], ((j + 1) / kStages) & 1, S))) break;
+          if (!(ok = wait_bar(&S->full[0][stn], phn, S))) break;
           tc_fence_after();
           mma_nt<D>(sbase, tmem, 0, 0, stn, 0);  // S_{j+1}
           mma_commit(&S->s_ready);
@@ -572,10 +594,13 @@ dq_kernel(const __grid_constant__ BwdParams p) {
         if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 256, 128, L::ring(st, 0, 0), j > 0);  // dQ
-        mma_commit(&S->empty[st]);
+        mma_commit(&S->empty[0][st]);  // K_j read for the last time
         if (j + 1 < n) {
+          if (!(ok = wait_bar(&S->full[1][stn], phn, S))) break;
+          tc_fence_after();
           mma_nt<D>(sbase, tmem, 128, 1, stn, 1);  // dP_{j+1}
           mma_commit(&S->dp_ready);
+          mma_commit(&S->empty[1][stn]);  // V_{j+1} read for the last time
         }
       }
       if (ok) mma_commit(&S->o_full);
