@@ -40,7 +40,21 @@ __device__ __forceinline__ void from_f(__nv_bfloat16& d, float x) {
 }
 
 // z and out may be the same buffer (in-place update): every element is read
-// and then written by the same thread.
+// and then written by the same thread.  Each thread keeps kUnroll groups of
+// loads in flight before it computes and stores, so that a few CTAs per SM
+// cover the HBM latency.
+constexpr int kUnroll = 4;
+
+template <typename T>
+__device__ __forceinline__ void update8(const Vec8<T>& zv,
+                                        const Vec8<__nv_bfloat16>& vv,
+                                        float neg_sigma, Vec8<T>* dst) {
+  Vec8<T> o;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) o.set(e, fmaf(neg_sigma, vv.get(e), zv.get(e)));
+  *dst = o;
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256)
 one_step_kernel(const T* z, const __nv_bfloat16* __restrict__ v, T* out,
@@ -48,14 +62,26 @@ one_step_kernel(const T* z, const __nv_bfloat16* __restrict__ v, T* out,
   const int64_t n8 = n / 8;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  for (int64_t i = tid; i < n8; i += stride) {
-    const Vec8<T> zv = reinterpret_cast<const Vec8<T>*>(z)[i];
-    Vec8<__nv_bfloat16> vv;
-    vv.u = __ldcs(reinterpret_cast<const uint4*>(v) + i);
-    Vec8<T> o;
+  const Vec8<T>* z8 = reinterpret_cast<const Vec8<T>*>(z);
+  const uint4* v8 = reinterpret_cast<const uint4*>(v);
+  Vec8<T>* o8 = reinterpret_cast<Vec8<T>*>(out);
+  int64_t i = tid;
+  for (; i + (kUnroll - 1) * stride < n8; i += kUnroll * stride) {
+    Vec8<T> zv[kUnroll];
+    Vec8<__nv_bfloat16> vv[kUnroll];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) o.set(e, fmaf(neg_sigma, vv.get(e), zv.get(e)));
-    reinterpret_cast<Vec8<T>*>(out)[i] = o;
+    for (int u = 0; u < kUnroll; ++u) {
+      zv[u] = z8[i + u * stride];
+      vv[u].u = __ldcs(v8 + i + u * stride);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+      update8(zv[u], vv[u], neg_sigma, o8 + i + u * stride);
+  }
+  for (; i < n8; i += stride) {
+    Vec8<__nv_bfloat16> vv;
+    vv.u = __ldcs(v8 + i);
+    update8(z8[i], vv, neg_sigma, o8 + i);
   }
   for (int64_t i = n8 * 8 + tid; i < n; i += stride)  // fewer than 8 left
     from_f(out[i], fmaf(neg_sigma, __bfloat162float(v[i]), to_f(z[i])));
