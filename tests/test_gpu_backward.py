@@ -42,6 +42,12 @@ CASES = [
     WL.custom("aligned-W2", batch=1, heads=2, head_dim=128,
               tokens_per_frame=64, frames_per_chunk=2, num_chunks=7,
               window_chunks=2, seed=75),
+    # long rows and columns: 24 key tiles per dQ CTA and 24 query tiles per
+    # dK/dV CTA, so every streamed ring and ready barrier goes through a
+    # dozen phase flips (the other cases stop at a few)
+    WL.custom("long-W2", batch=1, heads=1, head_dim=128,
+              tokens_per_frame=1024, frames_per_chunk=1, num_chunks=6,
+              window_chunks=2, seed=76),
 ]
 
 
