@@ -103,6 +103,36 @@ def test_streamed_gpu_equals_oneshot_oracle(FV, w):
     err.check()
 
 
+# ---------------------------------------- closed form: uniform attention
+# With Q = 0 every visible score is 0, so P is exactly 1 on the visible keys
+# of Eq. 1: O_i is the mean of V over them and the log-sum-exp is the log of
+# their count, for the streamed and the one-shot path alike (no oracle).
+# O = (sum of V) / n accumulates in fp32 and is rounded to bf16 once, so
+# 1e-3 absolute covers it with room; the LSE is exact to fp32 rounding.
+UNIFORM = [SMALL[0], SMALL[1], SMALL[2], SMALL[6]]
+
+
+@pytest.mark.parametrize("w", UNIFORM, ids=lambda w: w.name)
+def test_uniform_attention_closed_form(FV, w):
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    vs, qs, ks, vts, want_all = [], [], [], [], []
+    for c, q, k, v in WL.chunk_stream(w):
+        zq = torch.zeros_like(q)
+        att.append(k.cuda(), v.cuda())
+        o, lse = att.forward(zq.cuda(), want_lse=True)
+        vs.append(to64(v))
+        lo = 0 if w.window_chunks < 0 else max(0, c - w.window_chunks)
+        vis = np.concatenate(vs[lo:c + 1], axis=1)           # [B, Lk, H, d]
+        want = np.broadcast_to(vis.mean(axis=1, keepdims=True), q.shape)
+        assert np.abs(to64(o.cpu()) - want).max() <= 1e-3, c
+        assert np.abs(lse.cpu().double().numpy() - np.log(vis.shape[1])).max() <= 1e-5, c
+        qs.append(zq), ks.append(k), vts.append(v), want_all.append(want)
+    o1 = FV.blockcausal_attention(FV.config_from_workload(w),
+                                  torch.cat(qs, 1).cuda(), torch.cat(ks, 1).cuda(),
+                                  torch.cat(vts, 1).cuda())
+    assert np.abs(to64(o1.cpu()) - np.concatenate(want_all, axis=1)).max() <= 1e-3
+
+
 def test_forward_is_deterministic_and_repeatable(FV):
     w = SMALL[1]
     att = FV.StreamingAttention(FV.config_from_workload(w))
