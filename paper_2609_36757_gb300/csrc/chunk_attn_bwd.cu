@@ -252,7 +252,7 @@ __device__ __forceinline__ void mma_nt(uint32_t sbase, uint32_t tmem, int c0,
 #pragma unroll
   for (int ks = 0; ks < D / 16; ++ks) {
     const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
-    mma_ss_w(tmem + c0, a_lo + off, b_lo + off, hi, kIdesc, ks > 0);
+    mma_ss(tmem + c0, a_lo + off, b_lo + off, hi, kIdesc, ks > 0);
   }
 }
 
@@ -268,7 +268,7 @@ __device__ __forceinline__ void mma_tn(uint32_t sbase, uint32_t tmem, int c0,
   const uint32_t b_lo = desc_lo(sbase + b_off, kBox);
 #pragma unroll
   for (int kk = 0; kk < kT / 16; ++kk)
-    mma_ts_w(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
+    mma_ts(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
              b_lo + (uint32_t)(kk * 2048 >> 4), hi, kIdesc, (acc | kk) != 0);
 }
 

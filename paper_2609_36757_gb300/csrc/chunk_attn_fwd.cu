@@ -293,7 +293,7 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
       const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
-      mma_ss_w(tmem + t * 128, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
+      mma_ss(tmem + t * 128, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
     }
   };
   // O_t += P_t V: P_t from TMEM (8 columns per 16 keys), V MN-major (d
@@ -303,7 +303,7 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     const uint32_t b0 = v_lo + (uint32_t)st * kStage16;
 #pragma unroll
     for (int kk = 0; kk < kBN / 16; ++kk)
-      mma_ts_w(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
+      mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
                b0 + (uint32_t)(kk * 2048 >> 4), hi, kIdescPV, (acc | kk) != 0);
   };
 

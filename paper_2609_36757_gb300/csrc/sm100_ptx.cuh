@@ -14,11 +14,6 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
-__device__ __forceinline__ uint32_t lane_id() {
-  uint32_t l;
-  asm volatile("mov.u32 %0, %%laneid;" : "=r"(l));
-  return l;
-}
 
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
@@ -37,9 +32,6 @@ __device__ __forceinline__ void fence_barrier_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile(
@@ -145,17 +137,6 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
       : "r"(taddr));
 }
 
-// 32 lanes x 32 bits, 16 consecutive columns.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]),
-        "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]),
-        "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-        "=r"(r[15])
-      : "r"(taddr));
-}
 
 __device__ __forceinline__ void tmem_st16(uint32_t taddr,
                                           const uint32_t (&r)[16]) {
@@ -192,26 +173,14 @@ __device__ __forceinline__ void tmem_wait_st() {
 }
 
 // ------------------------------------------------------------- tcgen05.mma
-// Shared-memory matrix descriptor (tcgen05 format): start address, leading
-// and stride byte offsets (16-byte units), descriptor version 1 at bit 46,
-// swizzle mode in bits 61-63 (2 = 128-byte swizzle).
-__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr,
-                                                    uint32_t lbo_bytes,
-                                                    uint32_t sbo_bytes) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
-  d |= (uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
-// The same descriptor as two 32-bit words, for issue loops that precompute
-// it: the low word holds the start address and the leading byte offset, the
-// high word the stride byte offset, version and swizzle.  Moving the start
-// address within shared memory changes only the low word (the 14-bit field
-// cannot carry: shared addresses are below 256 KB).
+// Shared-memory matrix descriptor (tcgen05 format), 64 bits: start address
+// (16-byte units) in bits 0-13, leading byte offset (16-byte units) in bits
+// 16-29, stride byte offset in bits 32-45, descriptor version 1 at bit 46,
+// swizzle mode in bits 61-63 (2 = 128-byte swizzle).  It is formed as two
+// 32-bit words so that issue loops can precompute it: the low word holds the
+// start address and the leading byte offset, the high word the rest.
+// Moving the start address within shared memory changes only the low word
+// (the 14-bit field cannot carry: shared addresses are below 256 KB).
 __host__ __device__ constexpr uint32_t desc_lo(uint32_t saddr,
                                                uint32_t lbo_bytes) {
   return ((saddr >> 4) & 0x3FFFu) | (((lbo_bytes >> 4) & 0x3FFFu) << 16);
@@ -230,34 +199,10 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n,
          ((n >> 3) << 17) | ((m >> 4) << 24);
 }
 
-// D[tmem] (+)= A[smem] * B[smem]^T, issued by one thread.
-__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t a_desc,
-                                       uint64_t b_desc, uint32_t idesc,
-                                       uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
-          d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// D[tmem] (+)= A[tmem] * B[smem], issued by one thread.
-__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem,
-                                       uint64_t b_desc, uint32_t idesc,
-                                       uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(
-          d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// mma_ss / mma_ts with the descriptors given as (low, high) words.
-__device__ __forceinline__ void mma_ss_w(uint32_t d_tmem, uint32_t a_lo,
+// D[tmem] (+)= A * B, issued by one thread; shared-memory operands are given
+// by their descriptor words.  mma_ss: A and B in shared memory; mma_ts: A in
+// TMEM (M rows on the lanes), B in shared memory.
+__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint32_t a_lo,
                                          uint32_t b_lo, uint32_t hi,
                                          uint32_t idesc, uint32_t accumulate) {
   asm volatile(
@@ -270,7 +215,7 @@ __device__ __forceinline__ void mma_ss_w(uint32_t d_tmem, uint32_t a_lo,
       "r"(a_lo), "r"(b_lo), "r"(hi), "r"(idesc), "r"(accumulate)
       : "memory");
 }
-__device__ __forceinline__ void mma_ts_w(uint32_t d_tmem, uint32_t a_tmem,
+__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem,
                                          uint32_t b_lo, uint32_t hi,
                                          uint32_t idesc, uint32_t accumulate) {
   asm volatile(
