@@ -94,14 +94,24 @@ struct Work {
   int kv0, kv1;  // one-shot: the unit's key token range [kv0, kv1)
 };
 
-// One-shot launches: unit x covers query pair nq - 1 - x / (H B) of head
-// x % H, batch (x / H) % B, so the units with the most keys start first.
-// Its keys are the union of what its rows see: chunks max(0, c_lo - W) ..
-// c_hi of the unit's first and last rows (Eq. 1 with window W).
+// One-shot launches: the query pairs are grouped from the end of the
+// sequence into blocks of kOneShotBlock pairs; unit x takes block
+// x / (kOneShotBlock H B) (the units with the most keys start first), then
+// (b, h) and a pair within the block with the pair fastest, so that the CTAs
+// of one wave stream the keys of a few heads, each shared by up to
+// kOneShotBlock CTAs, rather than of every head at once.  A unit's keys are
+// the union of what its rows see: chunks max(0, c_lo - W) .. c_hi of its
+// first and last rows (Eq. 1 with window W).
+constexpr int kOneShotBlock = 32;
+
 __device__ __forceinline__ Work oneshot_work(const TcParams& p) {
   Work w;
-  const int bh = blockIdx.x % (p.heads * p.batch);
-  const int pair = p.q_pairs - 1 - blockIdx.x / (p.heads * p.batch);
+  const int hb = p.heads * p.batch;
+  const int blk = blockIdx.x / (kOneShotBlock * hb);
+  const int x = blockIdx.x % (kOneShotBlock * hb);
+  const int in_blk = min(kOneShotBlock, p.q_pairs - blk * kOneShotBlock);
+  const int bh = x / in_blk;
+  const int pair = p.q_pairs - 1 - blk * kOneShotBlock - x % in_blk;
   w.h = bh % p.heads;
   w.b = bh / p.heads;
   w.q0 = pair * kQTiles * kBM;
