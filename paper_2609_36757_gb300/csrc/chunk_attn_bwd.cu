@@ -683,34 +683,57 @@ dq_kernel(const __grid_constant__ BwdParams p) {
 // minus the forward LSE in log2 units (negated so that both enter packed
 // FMAs as addends), each [B*H, Lpad] with Lpad = L rounded up to 128 and
 // zeros in the padding (so every 128-token slice is aligned and in bounds).
-// One warp per (b, token, head) row of O.
+// D / 8 lanes per (b, token, head) row of O (one 16-byte piece each), so a
+// warp reads 32 / (D / 8) adjacent rows per instruction, and each lane keeps
+// kDeltaUnroll such row groups in flight.
+constexpr int kDeltaUnroll = 4;
+
 template <int D>
 __global__ void __launch_bounds__(256)
 delta_kernel(const uint16_t* o, const uint16_t* dO, const float* lse,
              float* lse2, float* delta, int batch, int heads, int seq,
              int padded) {
+  constexpr int kLanesPerRow = D / 8;
+  constexpr int kRowsPerWarp = 32 / kLanesPerRow;
   const int64_t rows = (int64_t)batch * seq * heads;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
   const int lane = threadIdx.x % 32;
+  const int sub = lane / kLanesPerRow, piece = lane % kLanesPerRow;
   const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
-  for (int64_t r = warp; r < rows; r += nwarps) {  // r = (b, token, head)
-    float acc = 0.f;
-    for (int x = lane * 2; x < D; x += 64) {
-      const __nv_bfloat162 a =
-          *reinterpret_cast<const __nv_bfloat162*>(o + r * D + x);
-      const __nv_bfloat162 g =
-          *reinterpret_cast<const __nv_bfloat162*>(dO + r * D + x);
-      acc = fmaf(__low2float(a), __low2float(g), acc);
-      acc = fmaf(__high2float(a), __high2float(g), acc);
+  const int64_t step = nwarps * kRowsPerWarp;  // rows between a lane's groups
+  for (int64_t r0 = warp * kRowsPerWarp; r0 < rows; r0 += step * kDeltaUnroll) {
+    uint4 a[kDeltaUnroll], g[kDeltaUnroll];
+#pragma unroll
+    for (int u = 0; u < kDeltaUnroll; ++u) {
+      const int64_t r = r0 + u * step + sub;  // r = (b, token, head)
+      a[u] = g[u] = make_uint4(0, 0, 0, 0);
+      if (r < rows) {
+        a[u] = __ldcs(reinterpret_cast<const uint4*>(o + r * D) + piece);
+        g[u] = __ldcs(reinterpret_cast<const uint4*>(dO + r * D) + piece);
+      }
     }
 #pragma unroll
-    for (int m = 16; m > 0; m >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, m);
-    if (lane == 0) {
-      const int64_t h = r % heads, bt = r / heads;
-      const int64_t tok = bt % seq, b = bt / seq;
-      const int64_t i = (b * heads + h) * padded + tok;
-      delta[i] = -acc;
-      lse2[i] = -lse[(b * heads + h) * seq + tok] * 1.4426950408889634f;
+    for (int u = 0; u < kDeltaUnroll; ++u) {
+      const uint32_t* ap = reinterpret_cast<const uint32_t*>(&a[u]);
+      const uint32_t* gp = reinterpret_cast<const uint32_t*>(&g[u]);
+      float acc = 0.f;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        acc = fmaf(__uint_as_float(ap[e] << 16), __uint_as_float(gp[e] << 16), acc);
+        acc = fmaf(__uint_as_float(ap[e] & 0xffff0000u),
+                   __uint_as_float(gp[e] & 0xffff0000u), acc);
+      }
+#pragma unroll
+      for (int m = kLanesPerRow / 2; m > 0; m >>= 1)
+        acc += __shfl_xor_sync(0xffffffffu, acc, m);
+      const int64_t r = r0 + u * step + sub;
+      if (piece == 0 && r < rows) {
+        const int64_t h = r % heads, bt = r / heads;
+        const int64_t tok = bt % seq, b = bt / seq;
+        const int64_t i = (b * heads + h) * padded + tok;
+        delta[i] = -acc;
+        lse2[i] = -lse[(b * heads + h) * seq + tok] * 1.4426950408889634f;
+      }
     }
   }
   // padding tokens
