@@ -28,6 +28,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "fastvr_internal.h"
 #include "sm100_ptx.cuh"
@@ -785,6 +786,36 @@ bool token_major_map(CUtensorMap* m, const void* base, int d, int L, int H,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// One non-blocking side stream and a fork / join event pair per device,
+// created on first use and kept until exit.  Calls on one device share them:
+// the caller holds g_side_mutex from the fork record to the join wait, so
+// host threads cannot interleave their event records, and their dQ kernels
+// run one after the other on the side stream.
+struct SideStream {
+  cudaStream_t stream;
+  cudaEvent_t fork, join;
+};
+constexpr int kMaxSideDevices = 64;
+std::mutex g_side_mutex;
+SideStream* g_side[kMaxSideDevices] = {};
+
+// Requires g_side_mutex held.
+SideStream* side_stream(int dev) {
+  if (dev < 0 || dev >= kMaxSideDevices) return nullptr;
+  if (g_side[dev] == nullptr) {
+    SideStream* s = new SideStream();
+    if (cudaStreamCreateWithFlags(&s->stream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&s->fork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&s->join, cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      delete s;
+      return nullptr;
+    }
+    g_side[dev] = s;
+  }
+  return g_side[dev];
+}
+
 template <int D>
 cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   BwdParams p;
@@ -828,6 +859,30 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int grid = p.tiles * a.heads * a.batch;
+  // dK/dV and dQ are independent (both read only the inputs and the
+  // scratch rows).  With few waves, dQ runs on a side stream forked after
+  // delta_kernel and joined before return, so its CTAs fill the SMs that
+  // dK/dV's last, partial wave leaves idle (training clip, 15 waves: +1.7 %);
+  // with many waves the tail is negligible and two long-sequence kernels at
+  // once contend for L2 (1080p sequence, 151 waves: -2 %), so both run in
+  // order, as they also do without a side stream.
+  constexpr int kMaxForkWaves = 32;
+  std::lock_guard<std::mutex> lock(g_side_mutex);
+  SideStream* side = grid <= kMaxForkWaves * (sms > 0 ? sms : 152)
+                         ? side_stream(dev)
+                         : nullptr;
+  if (side != nullptr && cudaEventRecord(side->fork, stream) == cudaSuccess &&
+      cudaStreamWaitEvent(side->stream, side->fork, 0) == cudaSuccess) {
+    dkdv_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+    dq_kernel<D><<<grid, kThreads, smem, side->stream>>>(p);
+    e = cudaGetLastError();
+    const cudaError_t j = cudaEventRecord(side->join, side->stream);
+    const cudaError_t w = j == cudaSuccess
+                              ? cudaStreamWaitEvent(stream, side->join, 0)
+                              : j;
+    return e != cudaSuccess ? e : w;
+  }
+  cudaGetLastError();
   dkdv_kernel<D><<<grid, kThreads, smem, stream>>>(p);
   dq_kernel<D><<<grid, kThreads, smem, stream>>>(p);
   return cudaGetLastError();
