@@ -27,7 +27,8 @@
  *    in fastvr_get_status.
  *  - Errors are returned as status codes; nothing throws or aborts across the
  *    ABI.  A call that returns an error enqueues no work and leaves the plan's
- *    counters unchanged.  Device-side failures (a bounded wait that gave up)
+ *    counters unchanged.  Device-side failures (a bounded wait that gave up;
+ *    in the debug library also a failed index check)
  *    are recorded in the cache's control word and reported by
  *    fastvr_get_status.
  *  - There is no CPU fallback: on a device that is not sm_103 the first
@@ -61,7 +62,9 @@ typedef enum {
   FASTVR_ERR_SEQUENCE = 4,     /* fwd before any append; append after a
                                   ragged (final) chunk                        */
   FASTVR_ERR_CUDA = 5,         /* a CUDA runtime/driver call failed           */
-  FASTVR_ERR_TIMEOUT = 6       /* a bounded device-side wait gave up          */
+  FASTVR_ERR_TIMEOUT = 6,      /* a bounded device-side wait gave up          */
+  FASTVR_ERR_BOUNDS = 7        /* debug library only: a device-side index
+                                  check failed and the access was skipped     */
 } fastvr_status_t;
 
 typedef struct {
@@ -264,6 +267,20 @@ FASTVR_API fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t plan,
 FASTVR_API fastvr_status_t fastvr_debug_inject_stall(fastvr_plan_t plan,
                                                      int32_t stall,
                                                      uint64_t wait_limit_ns);
+
+/* Index-check hook (tests of the debug library).  The debug library,
+ * libfastvr_attn_debug.so (built with FASTVR_BOUNDS_CHECK), checks every
+ * computed global-memory index of the append and attention kernels before
+ * the access; a failed check skips the access and records
+ * FASTVR_ERR_BOUNDS for fastvr_get_status.  This call makes the next
+ * fastvr_kv_append of the plan write its chunk `tokens` cache tokens past
+ * the start of its slot (0 <= tokens <= k * N), a deliberately wrong
+ * destination for those checks to catch: every write they let through
+ * stays inside the plan's cache buffer.  The cache contents are undefined
+ * afterwards (reset the plan).  Host only.  Errors: INVALID_ARG (tokens out
+ * of range), UNSUPPORTED (the release library, which has no checks). */
+FASTVR_API fastvr_status_t fastvr_debug_shift_next_append(fastvr_plan_t plan,
+                                                          int64_t tokens);
 
 /* Release a plan (host memory only; the cache stays the caller's). */
 FASTVR_API void fastvr_plan_destroy(fastvr_plan_t plan);

@@ -19,6 +19,10 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfastvr_attn.so")
+# The debug variant: every computed global index of the append and attention
+# kernels is checked before the access (FASTVR_BOUNDS_CHECK).
+DEBUG_BUILD = os.path.join(HERE, "_build_debug")
+DEBUG_LIB = os.path.join(HERE, "libfastvr_attn_debug.so")
 INCLUDE = os.path.join(ROOT, "include")
 
 SOURCES = ["fastvr_host.cpp", "kv_append.cu", "chunk_attn_fwd.cu",
@@ -50,8 +54,8 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def _compile(nvcc: str, src: str, force: bool, extra) -> str:
-    obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
+def _compile(nvcc: str, src: str, force: bool, extra, build_dir: str) -> str:
+    obj = os.path.join(build_dir, os.path.splitext(src)[0] + ".o")
     path = os.path.join(CSRC, src)
     if force or _stale(obj, [path, __file__] + _headers()):
         cmd = [nvcc, "-c", path, "-o", obj] + ARCH + FLAGS + list(extra)
@@ -63,18 +67,33 @@ def _compile(nvcc: str, src: str, force: bool, extra) -> str:
     return obj
 
 
-def build(force: bool = False, verbose_ptxas: bool = False) -> str:
-    os.makedirs(BUILD, exist_ok=True)
-    nvcc = _nvcc()
-    extra = ["-Xptxas", "-v"] if verbose_ptxas else []
-    with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(lambda s: _compile(nvcc, s, force, extra), SOURCES))
-    if force or _stale(LIB, objs):
-        cmd = [nvcc, "-shared", "-o", LIB] + objs + ARCH + [
+def _link(nvcc: str, lib: str, objs, force: bool) -> None:
+    if force or _stale(lib, objs):
+        cmd = [nvcc, "-shared", "-o", lib] + objs + ARCH + [
             "-cudart", "static", "-Xcompiler", "-fPIC"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+
+
+def build(force: bool = False, verbose_ptxas: bool = False,
+          debug: bool = True) -> str:
+    """Build the release library (and, with debug, the index-checking one:
+    both compile in one parallel pool).  Returns the release library path."""
+    nvcc = _nvcc()
+    extra = ["-Xptxas", "-v"] if verbose_ptxas else []
+    jobs = [(s, extra, BUILD) for s in SOURCES]
+    if debug:
+        jobs += [(s, extra + ["-DFASTVR_BOUNDS_CHECK"], DEBUG_BUILD)
+                 for s in SOURCES]
+    for d in {j[2] for j in jobs}:
+        os.makedirs(d, exist_ok=True)
+    with cf.ThreadPoolExecutor(max_workers=len(jobs)) as ex:
+        objs = list(ex.map(lambda j: _compile(nvcc, j[0], force, j[1], j[2]),
+                           jobs))
+    _link(nvcc, LIB, objs[:len(SOURCES)], force)
+    if debug:
+        _link(nvcc, DEBUG_LIB, objs[len(SOURCES):], force)
     return LIB
 
 

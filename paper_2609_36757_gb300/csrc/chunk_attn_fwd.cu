@@ -80,6 +80,8 @@ struct TcParams {
   int32_t q_pairs, units_full, split;
   float* ws;      // partial O: [part][d][kUnitRows]
   float* ws_lse;  // partial log2-domain LSE: [part][kUnitRows]
+  int32_t ws_parts;  // partial results the workspace holds
+  int64_t o_elems;   // elements of o (B Lq H d), for the debug index checks
   // One-shot (training-form) launches: the whole sequence of seq_tokens
   // tokens, chunks of chunk_tokens tokens, window W (-1: unbounded).
   int32_t seq_tokens, chunk_tokens, window, batch;
@@ -562,10 +564,16 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
       tmem_ld32(tO + c * 32, r);
       tmem_wait_ld();
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        ws_o[(c * 32 + i) * kUnitRows + r_unit] = __uint_as_float(r[i]) * inv_l;
+      for (int i = 0; i < 32; ++i) {
+        const int64_t x = (int64_t)w.part * D * kUnitRows +
+                          (int64_t)(c * 32 + i) * kUnitRows + r_unit;
+        if (in_bounds(x, (int64_t)p.ws_parts * D * kUnitRows, p.status))
+          ws_o[(c * 32 + i) * kUnitRows + r_unit] = __uint_as_float(r[i]) * inv_l;
+      }
     }
-    ws_l[r_unit] = m_ref + __log2f(l);
+    if (in_bounds((int64_t)w.part * kUnitRows + r_unit,
+                  (int64_t)p.ws_parts * kUnitRows, p.status))
+      ws_l[r_unit] = m_ref + __log2f(l);
     return;
   }
   const bool in_range = row < p.q_tokens;
@@ -586,12 +594,14 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
       uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
       for (int v = 0; v < 4; ++v)
-        dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        if (in_bounds(orow - p.o + c * 32 + 8 * v, p.o_elems - 7, p.status))
+          dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
     }
   }
-  if (p.lse != nullptr && in_range)
-    p.lse[((int64_t)w.b * p.heads + w.h) * p.q_tokens + row] =
-        (m_ref + __log2f(l)) * 0.6931471805599453f;
+  const int64_t lse_i = ((int64_t)w.b * p.heads + w.h) * p.q_tokens + row;
+  if (p.lse != nullptr && in_range &&
+      in_bounds(lse_i, (int64_t)p.batch * p.heads * p.q_tokens, p.status))
+    p.lse[lse_i] = (m_ref + __log2f(l)) * 0.6931471805599453f;
 }
 
 // Merge the partial results of the split units: weights 2^(lse_i - m),
@@ -618,6 +628,8 @@ combine_kernel(const __grid_constant__ TcParams p) {
   const int row0 = pair * kQTiles * kBM + blockIdx.y * kMergeRows;
   if (row0 >= p.q_tokens) return;  // the whole block is past the chunk end
   const int k0 = ut * p.split;
+  // every part this block reads lies in the workspace
+  if (!in_bounds(k0 + p.split - 1, p.ws_parts, p.status)) return;
   float m = -INFINITY;
   for (int i = 0; i < p.split; ++i)
     m = fmaxf(m, p.ws_lse[(size_t)(k0 + i) * kUnitRows + r_unit]);
@@ -641,18 +653,19 @@ combine_kernel(const __grid_constant__ TcParams p) {
   for (int x = 0; x < kCols; x += 2)
     *reinterpret_cast<uint32_t*>(&tile[r][g * kCols + x]) =
         pack_bf16(acc[x] * inv, acc[x + 1] * inv);
-  if (g == 0 && p.lse != nullptr && row0 + r < p.q_tokens)
-    p.lse[((int64_t)b * p.heads + h) * p.q_tokens + row0 + r] =
-        (m + __log2f(wsum)) * 0.6931471805599453f;
+  const int64_t lse_i = ((int64_t)b * p.heads + h) * p.q_tokens + row0 + r;
+  if (g == 0 && p.lse != nullptr && row0 + r < p.q_tokens &&
+      in_bounds(lse_i, (int64_t)p.batch * p.heads * p.q_tokens, p.status))
+    p.lse[lse_i] = (m + __log2f(wsum)) * 0.6931471805599453f;
   __syncthreads();
   // Each row is d bf16 = D / 8 16-byte pieces; one piece per thread.
   for (int i = threadIdx.x; i < kMergeRows * D / 8; i += blockDim.x) {
     const int rr = i / (D / 8), piece = i % (D / 8);
     const int row = row0 + rr;
-    if (row < p.q_tokens)
-      *reinterpret_cast<uint4*>(p.o + (int64_t)b * p.o_str.batch +
-                                (int64_t)row * p.o_str.token +
-                                (int64_t)h * p.o_str.head + piece * 8) =
+    const int64_t x = (int64_t)b * p.o_str.batch + (int64_t)row * p.o_str.token +
+                      (int64_t)h * p.o_str.head + piece * 8;
+    if (row < p.q_tokens && in_bounds(x, p.o_elems - 7, p.status))
+      *reinterpret_cast<uint4*>(p.o + x) =
           *reinterpret_cast<const uint4*>(&tile[rr][piece * 8]);
   }
 }
@@ -823,8 +836,11 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
   p.o = a.o;
   p.lse = a.lse;
   p.o_str = a.q_str;
+  p.o_elems = a.q_str.batch * a.batch;
   p.q_tokens = a.q_tokens;
   p.heads = a.heads;
+  p.batch = a.batch;
+  p.ws_parts = a.workspace_parts;
   p.scale_log2 = a.scale_log2;
   p.status = a.status;
   p.wait_limit_ns = a.wait_limit_ns;
@@ -874,6 +890,7 @@ cudaError_t launch_oneshot_d(const OneShotParams& a, cudaStream_t stream) {
   p.o_str.token = tok;
   p.o_str.head = D;
   p.o_str.batch = bat;
+  p.o_elems = bat * a.batch;
   p.q_tokens = a.seq_tokens;
   p.heads = a.heads;
   p.batch = a.batch;

@@ -47,6 +47,7 @@ struct fastvr_plan_s {
   int64_t launches;        // kernels enqueued since creation
   int32_t inject_stall;    // failure-detection test hook
   uint64_t wait_limit_ns;  // 0 = kernel default
+  int64_t append_shift;    // debug builds: next append's destination shift
 };
 
 namespace {
@@ -137,6 +138,7 @@ const char* fastvr_status_string(fastvr_status_t s) {
     case FASTVR_ERR_SEQUENCE: return "FASTVR_ERR_SEQUENCE";
     case FASTVR_ERR_CUDA: return "FASTVR_ERR_CUDA";
     case FASTVR_ERR_TIMEOUT: return "FASTVR_ERR_TIMEOUT";
+    case FASTVR_ERR_BOUNDS: return "FASTVR_ERR_BOUNDS";
   }
   return "FASTVR_ERR_UNKNOWN";
 }
@@ -216,7 +218,9 @@ fastvr_status_t fastvr_kv_append(fastvr_plan_t p, const void* k_new,
   a.heads = p->cfg.heads;
   a.head_dim = p->cfg.head_dim;
   a.cache_tokens = p->cache_tokens;
-  a.token_offset = (p->chunks % p->slots) * p->slot_tokens;
+  a.token_offset = (p->chunks % p->slots) * p->slot_tokens + p->append_shift;
+  a.status = control_word(p);
+  p->append_shift = 0;
   if (fastvr::launch_kv_append(a, reinterpret_cast<cudaStream_t>(stream)) !=
       cudaSuccess)
     return FASTVR_ERR_CUDA;
@@ -293,7 +297,7 @@ fastvr_status_t fastvr_get_status(fastvr_plan_t p) {
   if (word != fastvr::kDevOk) {
     const int zero = 0;
     cudaMemcpy(control_word(p), &zero, sizeof(int), cudaMemcpyHostToDevice);
-    return FASTVR_ERR_TIMEOUT;
+    return word == fastvr::kDevBounds ? FASTVR_ERR_BOUNDS : FASTVR_ERR_TIMEOUT;
   }
   return FASTVR_OK;
 }
@@ -500,6 +504,18 @@ fastvr_status_t fastvr_debug_inject_stall(fastvr_plan_t p, int32_t stall,
   p->inject_stall = stall != 0;
   p->wait_limit_ns = wait_limit_ns;
   return FASTVR_OK;
+}
+
+fastvr_status_t fastvr_debug_shift_next_append(fastvr_plan_t p,
+                                              int64_t tokens) {
+  if (p == nullptr || tokens < 0 || tokens > p->slot_tokens)
+    return FASTVR_ERR_INVALID_ARG;
+#ifdef FASTVR_BOUNDS_CHECK
+  p->append_shift = tokens;
+  return FASTVR_OK;
+#else
+  return FASTVR_ERR_UNSUPPORTED;
+#endif
 }
 
 void fastvr_plan_destroy(fastvr_plan_t p) { delete p; }

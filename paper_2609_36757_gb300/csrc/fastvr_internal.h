@@ -24,6 +24,27 @@ inline size_t workspace_bytes(int head_dim) {
 // Error codes a kernel writes into the cache's control block.
 constexpr int kDevOk = 0;
 constexpr int kDevTimeout = 1;
+constexpr int kDevBounds = 2;  // debug builds: an index check failed
+
+#ifdef __CUDACC__
+// Debug builds (-DFASTVR_BOUNDS_CHECK, libfastvr_attn_debug.so) check every
+// computed global-memory index of the streaming path before the access: an
+// index outside [0, n) records kDevBounds in the status word (the first
+// error wins) and the access is skipped.  Release builds compile the check
+// away.  compute-sanitizer is not available, and a trap or failed assert
+// would take the GPU down with it.
+#ifdef FASTVR_BOUNDS_CHECK
+__device__ __forceinline__ bool in_bounds(int64_t i, int64_t n, int* status) {
+  if (i >= 0 && i < n) return true;
+  if (status != nullptr) atomicCAS(status, kDevOk, kDevBounds);
+  return false;
+}
+#else
+__device__ __forceinline__ bool in_bounds(int64_t, int64_t, int*) {
+  return true;
+}
+#endif
+#endif
 
 // Strided view of a bfloat16 [B, L, H, d] token-major tensor or of a head-major
 // cache [B, H, L, d]: element (b, t, h, x) lives at
@@ -40,6 +61,7 @@ struct AppendParams {
   int32_t batch, tokens, heads, head_dim;
   int64_t cache_tokens;   // tokens per head in the cache (S * k * N)
   int64_t token_offset;   // first cache token of the destination slot
+  int* status;            // control block word (bounds checks), or null
 };
 
 struct AttnParams {

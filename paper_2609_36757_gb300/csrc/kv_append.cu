@@ -27,6 +27,11 @@ __device__ __forceinline__ int64_t cache_index(const AppendParams& p,
   const uint32_t bt = r / (uint32_t)p.heads;
   const uint32_t t = bt % (uint32_t)p.tokens;
   const uint32_t b = bt / (uint32_t)p.tokens;
+#ifdef FASTVR_BOUNDS_CHECK
+  // a destination token past this head's cache is out of bounds even when
+  // the flat index still lands inside the buffer
+  if (p.token_offset + t >= p.cache_tokens) return -1;
+#endif
   return (((int64_t)b * p.heads + h) * p.cache_tokens + p.token_offset + t) *
              VPR + vec;
 }
@@ -38,6 +43,7 @@ __global__ void __launch_bounds__(256) kv_append_kernel(AppendParams p) {
       reinterpret_cast<const uint4*>(blockIdx.y ? p.v_new : p.k_new);
   uint4* dst = reinterpret_cast<uint4*>(blockIdx.y ? p.v_cache : p.k_cache);
   const uint32_t n = (uint32_t)p.batch * p.tokens * p.heads * VPR;
+  const int64_t cache_vecs = (int64_t)p.batch * p.heads * p.cache_tokens * VPR;
   const uint32_t stride = gridDim.x * blockDim.x;
   uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   for (; i + (kUnroll - 1) * stride < n; i += kUnroll * stride) {
@@ -45,10 +51,15 @@ __global__ void __launch_bounds__(256) kv_append_kernel(AppendParams p) {
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) v[u] = __ldcs(src + i + u * stride);
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u)
-      dst[cache_index<VPR>(p, i + u * stride)] = v[u];
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t c = cache_index<VPR>(p, i + u * stride);
+      if (in_bounds(c, cache_vecs, p.status)) dst[c] = v[u];
+    }
   }
-  for (; i < n; i += stride) dst[cache_index<VPR>(p, i)] = __ldcs(src + i);
+  for (; i < n; i += stride) {
+    const int64_t c = cache_index<VPR>(p, i);
+    if (in_bounds(c, cache_vecs, p.status)) dst[c] = __ldcs(src + i);
+  }
 }
 
 }  // namespace

@@ -18,6 +18,8 @@ from typing import Optional, Tuple
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libfastvr_attn.so")
+# The same library with device-side index checks (FASTVR_BOUNDS_CHECK).
+DEBUG_LIB_PATH = os.path.join(_HERE, "libfastvr_attn_debug.so")
 
 FASTVR_OK = 0
 FASTVR_ERR_INVALID_ARG = 1
@@ -26,6 +28,7 @@ FASTVR_ERR_CAPACITY = 3
 FASTVR_ERR_SEQUENCE = 4
 FASTVR_ERR_CUDA = 5
 FASTVR_ERR_TIMEOUT = 6
+FASTVR_ERR_BOUNDS = 7
 
 
 class fastvr_attn_config_t(ctypes.Structure):
@@ -70,17 +73,18 @@ SIGNATURES = {
                                             ctypes.POINTER(_I64), _VP, _VP,
                                             _VP]),
     "fastvr_debug_inject_stall": (_I32, [_VP, _I32, ctypes.c_uint64]),
+    "fastvr_debug_shift_next_append": (_I32, [_VP, _I64]),
     "fastvr_plan_destroy": (None, [_VP]),
     "fastvr_status_string": (ctypes.c_char_p, [_I32]),
 }
 
 
-def _load() -> ctypes.CDLL:
-    if not os.path.exists(LIB_PATH):
+def _load(path: str = LIB_PATH) -> ctypes.CDLL:
+    if not os.path.exists(path):
         raise ImportError(
-            f"{LIB_PATH} is missing: build it with "
+            f"{path} is missing: build it with "
             "`python -m paper_2609_36757_gb300.build` (there is no fallback)")
-    lib = ctypes.CDLL(LIB_PATH)
+    lib = ctypes.CDLL(path)
     for name, (res, args) in SIGNATURES.items():
         fn = getattr(lib, name)
         fn.restype = res
@@ -89,6 +93,14 @@ def _load() -> ctypes.CDLL:
 
 
 lib = _load()
+
+
+def use_library(path: str) -> ctypes.CDLL:
+    """Route every call of this module to the library at path (e.g.
+    DEBUG_LIB_PATH) and return the one used before."""
+    global lib
+    previous, lib = lib, _load(path)
+    return previous
 
 
 class FastVRError(RuntimeError):
@@ -281,6 +293,11 @@ def fastvr_debug_inject_stall(plan: int, stall: int,
                               wait_limit_ns: int) -> None:
     _check(lib.fastvr_debug_inject_stall(plan, stall, wait_limit_ns),
            "fastvr_debug_inject_stall")
+
+
+def fastvr_debug_shift_next_append(plan: int, tokens: int) -> None:
+    _check(lib.fastvr_debug_shift_next_append(plan, tokens),
+           "fastvr_debug_shift_next_append")
 
 
 def fastvr_plan_destroy(plan: int) -> None:

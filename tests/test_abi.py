@@ -42,9 +42,40 @@ def test_every_declared_symbol_is_exported(fv):
     assert names == set(fv.SIGNATURES), "binding and header disagree"
 
 
+def test_debug_library_exports_the_same_symbols(fv):
+    names = _declared_symbols()
+    lib = ctypes.CDLL(fv.DEBUG_LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_append_shift_hook_exists_only_in_the_debug_library(fv):
+    cfg, plan = _plan(fv)
+    try:
+        with pytest.raises(fv.FastVRError) as e:
+            fv.fastvr_debug_shift_next_append(plan, 1)
+        assert e.value.status == fv.FASTVR_ERR_UNSUPPORTED
+        previous = fv.use_library(fv.DEBUG_LIB_PATH)
+        try:
+            dplan = fv.fastvr_attn_plan(cfg, FAKE, fv.fastvr_kv_cache_bytes(cfg))
+            try:
+                fv.fastvr_debug_shift_next_append(dplan, 8)  # one slot: k N
+                for bad in (-1, 9):
+                    with pytest.raises(fv.FastVRError) as e:
+                        fv.fastvr_debug_shift_next_append(dplan, bad)
+                    assert e.value.status == fv.FASTVR_ERR_INVALID_ARG
+            finally:
+                fv.fastvr_plan_destroy(dplan)
+        finally:
+            fv.lib = previous
+    finally:
+        fv.fastvr_plan_destroy(plan)
+
+
 def test_status_strings(fv):
     assert fv.fastvr_status_string(fv.FASTVR_OK) == "FASTVR_OK"
     assert fv.fastvr_status_string(fv.FASTVR_ERR_TIMEOUT) == "FASTVR_ERR_TIMEOUT"
+    assert fv.fastvr_status_string(fv.FASTVR_ERR_BOUNDS) == "FASTVR_ERR_BOUNDS"
     assert fv.fastvr_status_string(99) == "FASTVR_ERR_UNKNOWN"
 
 
