@@ -735,25 +735,6 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
 }
 
 // ------------------------------------------------------------------ host
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType,
-                                  cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*,
-                                  const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion,
-                                  CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  if (fn == nullptr) {
-    cudaDriverEntryPointQueryResult q;
-    void* ptr = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                         cudaEnableDefault, &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(ptr);
-  }
-  return fn;
-}
 
 // 4-D bf16 map over (x = d, token, head, batch) with a box of 64 x 128
 // (one 128-byte swizzled row per token); element strides in bytes.
@@ -793,7 +774,7 @@ int total_tiles(const AttnParams& a) {
 bool make_map(CUtensorMap* m, const void* base, int d, int64_t tokens,
               int heads, int batch, int64_t token_stride_b,
               int64_t head_stride_b, int64_t batch_stride_b) {
-  EncodeTiledFn enc = encode_fn();
+  EncodeTiledFn enc = encode_tiled_fn();
   if (enc == nullptr) return false;
   const cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)tokens,
                               (cuuint64_t)heads, (cuuint64_t)batch};
@@ -934,6 +915,22 @@ cudaError_t launch_chunk_attn(const AttnParams& p, cudaStream_t stream,
   if (p.head_dim == 64) return launch_d<64>(p, stream, launches);
   if (p.head_dim == 128) return launch_d<128>(p, stream, launches);
   return cudaErrorInvalidValue;
+}
+
+// Resolved once; C++ initialises the function-local static exactly once even
+// when several host threads make their first call at the same time.
+EncodeTiledFn encode_tiled_fn() {
+  static const EncodeTiledFn fn = []() -> EncodeTiledFn {
+    cudaDriverEntryPointQueryResult q;
+    void* ptr = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      return reinterpret_cast<EncodeTiledFn>(ptr);
+    cudaGetLastError();
+    return nullptr;
+  }();
+  return fn;
 }
 
 }  // namespace fastvr

@@ -2,6 +2,8 @@
 // CUDA kernels.  Not part of the public ABI.
 #pragma once
 
+#include <cuda.h>  // CUtensorMap types (the driver itself is reached
+                   // through the runtime's entry-point query)
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -20,6 +22,17 @@ constexpr int kUnitRows = 256;
 inline size_t workspace_bytes(int head_dim) {
   return (size_t)kMaxParts * kUnitRows * (head_dim + 1) * sizeof(float);
 }
+
+// cuTensorMapEncodeTiled, looked up through the CUDA runtime's driver entry
+// point (the library links the runtime statically and not libcuda); null
+// when the driver does not provide it.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType,
+                                  cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled_fn();
 
 // Error codes a kernel writes into the cache's control block.
 constexpr int kDevOk = 0;
