@@ -40,7 +40,11 @@ using namespace sm100;
 
 constexpr int kT = 128;           // tile rows (TMEM lanes) and tile columns
 constexpr int kBox = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (bytes)
-constexpr int kStages = 2;        // streamed-operand ring depth
+constexpr int kMaxStages = 3;     // deepest streamed ring
+constexpr int kStages1 = 2;       // ring 1 depth (ring 0: per kernel)
+constexpr int kDkdvS0 = 2;        // dK/dV ring 0 (Q and row vectors)
+constexpr int kDqS0 = 3;          // dQ ring 0 (K): loads one step earlier
+static_assert(kDkdvS0 == kStages1, "dK/dV indexes both rings alike");
 constexpr int kThreads = 320;     // 8 compute warps, producer, MMA issuer
 constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp = 9;
@@ -65,27 +69,35 @@ struct BwdShared {
   // vectors, read by dK), ring 1 the other (dq: V, last read by dP; dkdv:
   // dO, last read by dV), so a ring-1 slot is refilled as soon as its last
   // reader has run instead of waiting for the end of the step.
-  uint64_t full[2][kStages], empty[2][kStages];
+  uint64_t full[2][kMaxStages], empty[2][kMaxStages];
   uint64_t s_ready, dp_ready, p_ready, ds_ready, o_full, drain;
   uint32_t tmem_base;
   int abort;
-  // dkdv: the streamed query tile's -log2 LSE and -D, one slice per stage
-  __align__(16) float lse2[kStages][kT];
-  __align__(16) float dlt[kStages][kT];
 };
 
-template <int D>
+// Shared memory: the two fixed operands, ring 0 (kS0 stages), ring 1
+// (kStages1 stages), the barriers, and with kVecs the per-stage slices of
+// -log2 LSE and -D for ring 0's query tiles (dK/dV).  The dQ kernel's third
+// K stage fits only because it carries no slices.
+template <int D, int kS0, bool kVecs>
 struct BwdLayout {
+  static_assert(kS0 >= 2 && kS0 <= kMaxStages, "ring 0 depth");
   static constexpr int kNB = D / 64;
-  // fixed operands (two tiles), then the streamed ring of two tiles a stage
   __host__ __device__ static constexpr int fixed(int which, int bx) {
     return (which * kNB + bx) * kBox;
   }
   __host__ __device__ static constexpr int ring(int st, int which, int bx) {
-    return ((2 + st * 2 + which) * kNB + bx) * kBox;
+    return ((2 + (which ? kS0 + st : st)) * kNB + bx) * kBox;
   }
-  static constexpr int shared_off = (2 + 2 * kStages) * kNB * kBox;
-  static constexpr int bytes = shared_off + (int)sizeof(BwdShared) + 1024 + 64;
+  static constexpr int shared_off = (2 + kS0 + kStages1) * kNB * kBox;
+  static constexpr int vec_off =
+      shared_off + ((int)sizeof(BwdShared) + 15) / 16 * 16;
+  static constexpr int vec_bytes = kVecs ? 2 * kS0 * kT * (int)sizeof(float) : 0;
+  static constexpr int bytes = vec_off + vec_bytes + 1024 + 64;
+  // slice of stage st: lse2 at vec(0, st), dlt at vec(1, st) (floats)
+  __host__ __device__ static constexpr int vec(int which, int st) {
+    return vec_off + (which * kS0 + st) * kT * (int)sizeof(float);
+  }
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -155,7 +167,7 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
   if (threadIdx.x == kProducerWarp * 32) {
     mbar_init(&S->fixed_full, 1);
     for (int r = 0; r < 2; ++r)
-      for (int s = 0; s < kStages; ++s) {
+      for (int s = 0; s < kMaxStages; ++s) {
         mbar_init(&S->full[r][s], 1);
         mbar_init(&S->empty[r][s], 1);
       }
@@ -191,13 +203,13 @@ __device__ __forceinline__ void bwd_teardown(uint32_t tmem) {
 // streamed tiles per step (maps r0, r1 at token t0 + 128 j).
 // With kRowVecs, each step also bulk-copies the streamed tile's 128 log2-LSE
 // and D values (from the padded scratch rows vec_lse2, vec_dlt).
-template <int D, bool kRowVecs>
+template <int D, bool kRowVecs, int kS0>
 __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
                              const CUtensorMap* f1, int t_fixed,
                              const CUtensorMap* r0, const CUtensorMap* r1,
                              int t0, int n, int h, int b,
                              const float* vec_lse2, const float* vec_dlt) {
-  using L = BwdLayout<D>;
+  using L = BwdLayout<D, kS0, kRowVecs>;
   constexpr uint32_t kVecBytes = kRowVecs ? 2 * kT * sizeof(float) : 0;
   mbar_arrive_expect_tx(&S->fixed_full, 2 * L::kNB * kBox);
   for (int bx = 0; bx < L::kNB; ++bx) {
@@ -209,31 +221,31 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
   // follows.
   int issued[2] = {0, 0};
   for (int j = 0; j < n; ++j) {
-    const int st = j % kStages;
-    const uint32_t ph = ((j / kStages) & 1) ^ 1;
-    if (!wait_bar(&S->empty[1][st], ph, S)) break;
-    mbar_arrive_expect_tx(&S->full[1][st], L::kNB * kBox);
+    const int s1 = j % kStages1, s0 = j % kS0;
+    if (!wait_bar(&S->empty[1][s1], ((j / kStages1) & 1) ^ 1, S)) break;
+    mbar_arrive_expect_tx(&S->full[1][s1], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(r1, smem + L::ring(st, 1, bx), &S->full[1][st], bx * 64,
+      tma_load_4d(r1, smem + L::ring(s1, 1, bx), &S->full[1][s1], bx * 64,
                   t0 + j * kT, h, b);
     ++issued[1];
-    if (!wait_bar(&S->empty[0][st], ph, S)) break;
-    mbar_arrive_expect_tx(&S->full[0][st], L::kNB * kBox + kVecBytes);
+    if (!wait_bar(&S->empty[0][s0], ((j / kS0) & 1) ^ 1, S)) break;
+    mbar_arrive_expect_tx(&S->full[0][s0], L::kNB * kBox + kVecBytes);
     for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(r0, smem + L::ring(st, 0, bx), &S->full[0][st], bx * 64,
+      tma_load_4d(r0, smem + L::ring(s0, 0, bx), &S->full[0][s0], bx * 64,
                   t0 + j * kT, h, b);
     if (kRowVecs) {
-      bulk_load(S->lse2[st], vec_lse2 + t0 + j * kT, kT * sizeof(float),
-                &S->full[0][st]);
-      bulk_load(S->dlt[st], vec_dlt + t0 + j * kT, kT * sizeof(float),
-                &S->full[0][st]);
+      bulk_load(smem + L::vec(0, s0), vec_lse2 + t0 + j * kT, kT * sizeof(float),
+                &S->full[0][s0]);
+      bulk_load(smem + L::vec(1, s0), vec_dlt + t0 + j * kT, kT * sizeof(float),
+                &S->full[0][s0]);
     }
     ++issued[0];
   }
   drain_wait(&S->fixed_full, 0);
-  for (int r = 0; r < 2; ++r)
-    for (int i = max(0, issued[r] - kStages); i < issued[r]; ++i)
-      drain_wait(&S->full[r][i % kStages], (i / kStages) & 1);
+  for (int i = max(0, issued[1] - kStages1); i < issued[1]; ++i)
+    drain_wait(&S->full[1][i % kStages1], (i / kStages1) & 1);
+  for (int i = max(0, issued[0] - kS0); i < issued[0]; ++i)
+    drain_wait(&S->full[0][i % kS0], (i / kS0) & 1);
 }
 
 // One thread issues every MMA, and a tcgen05.mma takes it about as long to
@@ -242,10 +254,9 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
 // call and the K steps add constant offsets (16-byte units) to it.
 
 // D_t = A_fixed * B_ring^T over the head dim (both K-major): TMEM col c0.
-template <int D>
+template <int D, class L>
 __device__ __forceinline__ void mma_nt(uint32_t sbase, uint32_t tmem, int c0,
                                        int fixed_which, int st, int ring_which) {
-  using L = BwdLayout<D>;
   constexpr uint32_t kIdesc = idesc_bf16_f32(kT, kT, 0);
   const uint32_t hi = desc_hi_sw128(1024);
   const uint32_t a_lo = desc_lo(sbase + L::fixed(fixed_which, 0), 16);
@@ -377,7 +388,7 @@ __device__ __forceinline__ void ds32(const uint32_t (&pb)[16],
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 dkdv_kernel(const __grid_constant__ BwdParams p) {
-  using L = BwdLayout<D>;
+  using L = BwdLayout<D, kDkdvS0, true>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -401,7 +412,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
 
   if (warp == kProducerWarp) {
     if (lane == 0)
-      bwd_producer<D, true>(smem, S, &p.k_map, &p.v_map, k0, &p.q_map,
+      bwd_producer<D, true, kDkdvS0>(smem, S, &p.k_map, &p.v_map, k0, &p.q_map,
                             &p.do_map, q0, n, h, b,
                             p.lse2 + (int64_t)bh_row(p, b, h) * p.padded,
                             p.delta + (int64_t)bh_row(p, b, h) * p.padded);
@@ -418,14 +429,14 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
                 wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
       if (ok) {
         tc_fence_after();
-        mma_nt<D>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
+        mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
         mma_commit(&S->s_ready);
-        mma_nt<D>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
+        mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
         mma_commit(&S->dp_ready);
       }
       for (int j = 0; ok && j < n; ++j) {
-        const int st = j % kStages, stn = (j + 1) % kStages;
-        const uint32_t phn = ((j + 1) / kStages) & 1;
+        const int st = j % kStages1, stn = (j + 1) % kStages1;
+        const uint32_t phn = ((j + 1) / kStages1) & 1;
         if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
         tc_fence_after();
         mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
@@ -433,7 +444,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
         if (j + 1 < n) {
           if (!(ok = wait_bar(&S->full[0][stn], phn, S))) break;
           tc_fence_after();
-          mma_nt<D>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
+          mma_nt<D, L>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
           mma_commit(&S->s_ready);
         }
         if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
@@ -443,7 +454,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
         if (j + 1 < n) {
           if (!(ok = wait_bar(&S->full[1][stn], phn, S))) break;
           tc_fence_after();
-          mma_nt<D>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
+          mma_nt<D, L>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
           mma_commit(&S->dp_ready);
         }
       }
@@ -467,12 +478,13 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     bool ok = true;
     for (int j = 0; j < n; ++j) {
       const int i0 = q0 + j * kT + 64 * hf;  // first query of this half
-      const int st = j % kStages;
+      const int st = j % kDkdvS0;
       // the stage's LSE and D slices (the MMA warp frees the stage only after
       // ds_ready, so they stay valid while this tile is processed)
-      if (!(ok = wait_bar(&S->full[0][st], (j / kStages) & 1, S))) break;
-      const float* nl = S->lse2[st] + 64 * hf;  // -log2 LSE per column
-      const float* nd = S->dlt[st] + 64 * hf;   // -D per column
+      if (!(ok = wait_bar(&S->full[0][st], (j / kDkdvS0) & 1, S))) break;
+      // -log2 LSE and -D per column
+      const float* nl = reinterpret_cast<const float*>(smem + L::vec(0, st)) + 64 * hf;
+      const float* nd = reinterpret_cast<const float*>(smem + L::vec(1, st)) + 64 * hf;
       // the first half's LSE values land while S^T is computed
       float4 la[8], lb[8];
 #pragma unroll
@@ -545,7 +557,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 dq_kernel(const __grid_constant__ BwdParams p) {
-  using L = BwdLayout<D>;
+  using L = BwdLayout<D, kDqS0, false>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -564,7 +576,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
 
   if (warp == kProducerWarp) {
     if (lane == 0)
-      bwd_producer<D, false>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map,
+      bwd_producer<D, false, kDqS0>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map,
                              &p.v_map, kv0, n, h, b, nullptr, nullptr);
     __syncwarp();
   } else if (warp == kMmaWarp) {
@@ -576,32 +588,35 @@ dq_kernel(const __grid_constant__ BwdParams p) {
                 wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
       if (ok) {
         tc_fence_after();
-        mma_nt<D>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
+        mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
         mma_commit(&S->s_ready);
-        mma_nt<D>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
+        mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
         mma_commit(&S->dp_ready);
         mma_commit(&S->empty[1][0]);           // V_0 read for the last time
       }
       for (int j = 0; ok && j < n; ++j) {
-        const int st = j % kStages, stn = (j + 1) % kStages;
-        const uint32_t phn = ((j + 1) / kStages) & 1;
+        // K (ring 0) and V (ring 1) run at their own depths
+        const int k_st = j % kDqS0, k_stn = (j + 1) % kDqS0;
+        const int v_stn = (j + 1) % kStages1;
         if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
         if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[0][stn], phn, S))) break;
+          if (!(ok = wait_bar(&S->full[0][k_stn], ((j + 1) / kDqS0) & 1, S)))
+            break;
           tc_fence_after();
-          mma_nt<D>(sbase, tmem, 0, 0, stn, 0);  // S_{j+1}
+          mma_nt<D, L>(sbase, tmem, 0, 0, k_stn, 0);  // S_{j+1}
           mma_commit(&S->s_ready);
         }
         if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
         tc_fence_after();
-        mma_tn<D>(sbase, tmem, 256, 128, L::ring(st, 0, 0), j > 0);  // dQ
-        mma_commit(&S->empty[0][st]);  // K_j read for the last time
+        mma_tn<D>(sbase, tmem, 256, 128, L::ring(k_st, 0, 0), j > 0);  // dQ
+        mma_commit(&S->empty[0][k_st]);  // K_j read for the last time
         if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[1][stn], phn, S))) break;
+          if (!(ok = wait_bar(&S->full[1][v_stn], ((j + 1) / kStages1) & 1, S)))
+            break;
           tc_fence_after();
-          mma_nt<D>(sbase, tmem, 128, 1, stn, 1);  // dP_{j+1}
+          mma_nt<D, L>(sbase, tmem, 128, 1, v_stn, 1);  // dP_{j+1}
           mma_commit(&S->dp_ready);
-          mma_commit(&S->empty[1][stn]);  // V_{j+1} read for the last time
+          mma_commit(&S->empty[1][v_stn]);  // V_{j+1} read for the last time
         }
       }
       if (ok) mma_commit(&S->o_full);
@@ -832,12 +847,16 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   delta_kernel<D><<<(unsigned)blocks, 256, 0, stream>>>(
       a.out, a.dout, a.lse, a.scratch, a.scratch + (size_t)a.batch * a.heads * padded,
       a.batch, a.heads, L, padded);
-  const int smem = BwdLayout<D>::bytes;
+  const int smem = BwdLayout<D, kDkdvS0, true>::bytes;
+  const int smem_dq = BwdLayout<D, kDqS0, false>::bytes;
+  static_assert(BwdLayout<128, kDkdvS0, true>::bytes <= 227 * 1024 &&
+                    BwdLayout<128, kDqS0, false>::bytes <= 227 * 1024,
+                "backward shared memory");
   cudaError_t e = cudaFuncSetAttribute(
       dkdv_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(dq_kernel<D>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem_dq);
   if (e != cudaSuccess) return e;
   const int grid = p.tiles * a.heads * a.batch;
   // dK/dV and dQ are independent (both read only the inputs and the
@@ -855,7 +874,7 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   if (side != nullptr && cudaEventRecord(side->fork, stream) == cudaSuccess &&
       cudaStreamWaitEvent(side->stream, side->fork, 0) == cudaSuccess) {
     dkdv_kernel<D><<<grid, kThreads, smem, stream>>>(p);
-    dq_kernel<D><<<grid, kThreads, smem, side->stream>>>(p);
+    dq_kernel<D><<<grid, kThreads, smem_dq, side->stream>>>(p);
     e = cudaGetLastError();
     const cudaError_t j = cudaEventRecord(side->join, side->stream);
     const cudaError_t w = j == cudaSuccess
@@ -865,7 +884,7 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   }
   cudaGetLastError();
   dkdv_kernel<D><<<grid, kThreads, smem, stream>>>(p);
-  dq_kernel<D><<<grid, kThreads, smem, stream>>>(p);
+  dq_kernel<D><<<grid, kThreads, smem_dq, stream>>>(p);
   return cudaGetLastError();
 }
 
