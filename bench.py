@@ -454,29 +454,36 @@ def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
 
 def run_e2e(args, w, chunks, att, dev, step_flops, world):
     """The same metric through the public API from pinned host buffers: every
-    step copies each chunk's Q/K/V host->device (a side stream, overlapped
-    with the previous chunk's compute) and each output device->host."""
+    step copies each chunk's Q/K/V host->device and each output device->host,
+    on two side streams, through a ring of three device slots, so that a
+    chunk's inputs load while the previous chunk computes; the ring and its
+    events carry over from one step to the next, so the next step's first
+    chunk also loads while this step's last one computes."""
+    kSlots = 3
     pq = [q.pin_memory() for q, _, _ in chunks]
     pk = [k.pin_memory() for _, k, _ in chunks]
     pv = [v.pin_memory() for _, _, v in chunks]
     po = [torch.empty_like(q).pin_memory() for q in pq]
     slots = [[torch.empty_like(pq[0], device=dev) for _ in range(3)]
-             for _ in range(2)]
-    outs = [torch.empty_like(pq[0], device=dev) for _ in range(2)]
+             for _ in range(kSlots)]
+    outs = [torch.empty_like(pq[0], device=dev) for _ in range(kSlots)]
     compute = torch.cuda.current_stream(dev)
     h2d = torch.cuda.Stream(dev)
     d2h = torch.cuda.Stream(dev)
     h2d_bytes = sum(t.numel() * 2 for t in pq + pk + pv)
     d2h_bytes = sum(t.numel() * 2 for t in po)
+    # free[s]: the slot's inputs are consumed; out_free[s]: its output is out
+    free = [torch.cuda.Event() for _ in range(kSlots)]
+    out_free = [torch.cuda.Event() for _ in range(kSlots)]
+    for e in free + out_free:
+        e.record(compute)
+    used = [0]
 
     def step():
         att.reset()
-        free = [torch.cuda.Event(), torch.cuda.Event()]
-        out_free = [torch.cuda.Event(), torch.cuda.Event()]
-        for e in free + out_free:
-            e.record(compute)
         for c in range(w.num_chunks):
-            s = c % 2
+            s = used[0] % kSlots
+            used[0] += 1
             L = pq[c].shape[1]
             sq, sk, sv = (x[:, :L] for x in slots[s])
             with torch.cuda.stream(h2d):
@@ -498,7 +505,6 @@ def run_e2e(args, w, chunks, att, dev, step_flops, world):
                 d2h.wait_event(done)
                 po[c].copy_(o, non_blocking=True)
                 out_free[s].record(d2h)
-        compute.wait_stream(d2h)
 
     for _ in range(max(1, args.warmup)):
         step()
