@@ -1,0 +1,65 @@
+"""bench.py's JSON line: the keys and types the benchmark contract requires,
+for the reference arm (the oracle on the host; runs on CPU) and, on a GB300,
+for the library's own arm on a small workload."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _run(*args, timeout=600):
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), *args],
+                       cwd=ROOT, capture_output=True, text=True, timeout=timeout)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout[-2000:]
+    return json.loads(lines[0])
+
+
+def _common(d):
+    for k, t in (("metric", str), ("value", float), ("unit", str),
+                 ("n_gpus", int), ("steps", int), ("warmup", int),
+                 ("higher_is_better", bool), ("scaling", str), ("dtype", str),
+                 ("data", str), ("config", dict)):
+        assert isinstance(d[k], t), k
+    assert d["vs_baseline"] is None  # the paper reports no number for this path
+    assert d["config"]["workload"]
+    assert "model" not in d["config"]
+    assert d["value"] > 0
+    assert d["scaling"] == "weak" and d["higher_is_better"] is True
+
+
+def test_reference_arm_line():
+    d = _run("--impl", "reference", "--steps", "1", "--warmup", "1")
+    _common(d)
+    assert d["impl"] == "reference"
+    assert d["dtype"] == "f64"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"],
+                        "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+@pytest.mark.gpu
+def test_gpu_arm_line():
+    d = _run("--workload", "480p", "--steps", "3", "--warmup", "3",
+             "--cpu-seconds", "2")
+    _common(d)
+    assert d["n_gpus"] == 1 and d["steps"] == 3 and d["warmup"] == 3
+    assert d["dtype"] == "bf16"
+    assert d["ms_per_step"] > 0
+    r = d["roofline"]
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+    assert 0 < r["frac"] <= 1.2 and abs(r["frac"] - r["achieved"] / r["peak"]) < 1e-9
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] > 0
+    e = d["e2e"]
+    assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
+    # one append, one attention call and at most one merge per chunk and step
+    assert 2 * 8 * 3 <= d["gpu_launches"] <= 3 * 8 * 3
+    c = d["clocks"]
+    assert c["sm_max_mhz"] > 0 and isinstance(c["reasons"], list)
