@@ -162,7 +162,8 @@ FASTVR_API fastvr_status_t fastvr_plan_visible(fastvr_plan_t plan, int32_t* num_
  * block of 256 query rows reads only the keys its rows can see (invisible
  * chunks are never loaded); rows that straddle a chunk boundary are masked
  * element-wise.  No plan, no cache and no scratch memory are involved; a
- * bounded-wait timeout leaves out undefined and is not reported.  The result
+ * bounded-wait timeout leaves out undefined and is reported by
+ * fastvr_get_device_status.  The result
  * equals the streamed form (fastvr_kv_append + fastvr_chunk_attn_fwd, chunk
  * by chunk) up to rounding.
  * Errors: INVALID_ARG, UNSUPPORTED (head_dim, device not sm_103), CUDA. */
@@ -188,7 +189,7 @@ FASTVR_API fastvr_status_t fastvr_blockcausal_bwd_scratch_bytes(
  * tiles that see them) and dq (one CTA per 128 queries); P is recomputed
  * from lse, P and dS enter the tensor cores in bfloat16, accumulation is
  * fp32.  All pointers 16-byte aligned.  A bounded-wait timeout leaves the
- * outputs undefined and is not reported.
+ * outputs undefined and is reported by fastvr_get_device_status.
  * Errors: INVALID_ARG, UNSUPPORTED, CAPACITY (scratch too small), CUDA. */
 FASTVR_API fastvr_status_t fastvr_blockcausal_attn_bwd(
     const fastvr_attn_config_t* cfg, int32_t num_frames, const void* q,
@@ -267,6 +268,27 @@ FASTVR_API fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t plan,
 FASTVR_API fastvr_status_t fastvr_debug_inject_stall(fastvr_plan_t plan,
                                                      int32_t stall,
                                                      uint64_t wait_limit_ns);
+
+/* Device-side failures of the calls without a plan (the one-shot forward
+ * fastvr_blockcausal_attn_fwd and the backward fastvr_blockcausal_attn_bwd):
+ * a bounded wait that gave up — or, in the debug library, a failed index
+ * check — is recorded in a status word of the current device, shared by all
+ * such calls on it.  This call waits for the device to finish (it
+ * synchronises), returns FASTVR_ERR_TIMEOUT or FASTVR_ERR_BOUNDS for a
+ * recorded failure and clears the word, FASTVR_OK otherwise.  The outputs
+ * of a call that failed this way are undefined.  Errors: CUDA. */
+FASTVR_API fastvr_status_t fastvr_get_device_status(void);
+
+/* Failure-detection hook (tests) for the calls without a plan, process-wide:
+ * stall != 0 makes every following one-shot forward and backward launch
+ * wait, in its MMA-issuing thread, on a barrier that nothing arrives on; the
+ * bounded wait runs out after wait_limit_ns (0 = the 4 s default), every
+ * role stops, in-flight copies and MMAs are drained, tensor memory is
+ * released and FASTVR_ERR_TIMEOUT is recorded for fastvr_get_device_status.
+ * No GPU fault or hang results.  stall = 0 restores normal operation.
+ * Host only; always FASTVR_OK. */
+FASTVR_API fastvr_status_t fastvr_debug_inject_stall_noplan(
+    int32_t stall, uint64_t wait_limit_ns);
 
 /* Index-check hook (tests of the debug library).  The debug library,
  * libfastvr_attn_debug.so (built with FASTVR_BOUNDS_CHECK), checks every

@@ -60,6 +60,9 @@ struct BwdParams {
   uint16_t* dv;
   int32_t seq_tokens, heads, batch, chunk_tokens, window, tiles, padded;
   float scale, scale_log2;
+  int* status;             // device status word (timeouts) or null
+  int32_t inject_stall;    // test hook: the MMA thread waits on o_full first
+  uint64_t wait_limit_ns;  // 0 = kWaitLimitNs
 };
 
 struct BwdShared {
@@ -73,6 +76,8 @@ struct BwdShared {
   uint64_t s_ready, dp_ready, p_ready, ds_ready, o_full, drain;
   uint32_t tmem_base;
   int abort;
+  int* status;
+  uint64_t wait_limit_ns;
 };
 
 // Shared memory: the two fixed operands, ring 0 (kS0 stages), ring 1
@@ -118,8 +123,9 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*reinterpret_cast<volatile int*>(&S->abort)) return false;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
+    if (global_timer_ns() - t0 > S->wait_limit_ns) {
       *reinterpret_cast<volatile int*>(&S->abort) = 1;
+      if (S->status != nullptr) atomicExch(S->status, kDevTimeout);
       return false;
     }
   }
@@ -158,7 +164,8 @@ __device__ __forceinline__ void query_sees(const BwdParams& p, int row, int& lo,
 }
 
 // Common CTA prologue: TMEM (MMA warp) and barriers (producer thread).
-__device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
+__device__ __forceinline__ uint32_t bwd_setup(BwdShared* S,
+                                              const BwdParams& p) {
   const int warp = threadIdx.x / 32;
   if (warp == kMmaWarp) {
     tmem_alloc(&S->tmem_base, kTmemCols);
@@ -182,6 +189,8 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S) {
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
+    S->status = p.status;
+    S->wait_limit_ns = p.wait_limit_ns ? p.wait_limit_ns : kWaitLimitNs;
     fence_barrier_init();
   }
   tc_fence_before();
@@ -408,7 +417,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
                                         p.chunk_tokens,
                                     p.seq_tokens);
   const int n = (q1 - q0 + kT - 1) / kT;
-  const uint32_t tmem = bwd_setup(S);
+  const uint32_t tmem = bwd_setup(S, p);
 
   if (warp == kProducerWarp) {
     if (lane == 0)
@@ -425,7 +434,10 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       // the compute warps keep P^T in registers), and the next dP^T right
       // after dK (over dS^T), so the compute warps start the next tile's P
       // as soon as they finish this tile's dS.
-      bool ok = wait_bar(&S->fixed_full, 0, S) &&
+      // Test hook: o_full receives no arrival before the end, so this wait
+      // runs out and exercises the abort path.
+      bool ok = (!p.inject_stall || wait_bar(&S->o_full, 0, S)) &&
+                wait_bar(&S->fixed_full, 0, S) &&
                 wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
       if (ok) {
         tc_fence_after();
@@ -572,7 +584,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
   const int kv0 = p.window < 0 ? 0 : max(0, c_lo - p.window) * p.chunk_tokens;
   const int kv1 = min((c_hi + 1) * p.chunk_tokens, p.seq_tokens);
   const int n = (kv1 - kv0 + kT - 1) / kT;
-  const uint32_t tmem = bwd_setup(S);
+  const uint32_t tmem = bwd_setup(S, p);
 
   if (warp == kProducerWarp) {
     if (lane == 0)
@@ -584,7 +596,10 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       const uint32_t sbase = smem_addr(smem);
       // S of the next tile is issued as soon as P of this one is in
       // registers, so it overlaps the dS computation.
-      bool ok = wait_bar(&S->fixed_full, 0, S) &&
+      // Test hook: o_full receives no arrival before the end, so this wait
+      // runs out and exercises the abort path.
+      bool ok = (!p.inject_stall || wait_bar(&S->o_full, 0, S)) &&
+                wait_bar(&S->fixed_full, 0, S) &&
                 wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
       if (ok) {
         tc_fence_after();
@@ -837,6 +852,9 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   p.tiles = (L + kT - 1) / kT;
   p.scale = a.scale;
   p.scale_log2 = a.scale * 1.4426950408889634f;
+  p.status = a.status;
+  p.inject_stall = a.inject_stall;
+  p.wait_limit_ns = a.wait_limit_ns;
 
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);

@@ -877,6 +877,8 @@ cudaError_t launch_oneshot_d(const OneShotParams& a, cudaStream_t stream) {
   p.batch = a.batch;
   p.scale_log2 = a.scale_log2;
   p.status = a.status;
+  p.inject_stall = a.inject_stall;
+  p.wait_limit_ns = a.wait_limit_ns;
   p.seq_tokens = a.seq_tokens;
   p.chunk_tokens = a.chunk_tokens;
   p.window = a.window;

@@ -55,7 +55,29 @@ unsigned char* scratch_on_current_device(int dev) {
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+// The status word of the calls without a plan, one per device.
+static __device__ int g_device_status;
+int* g_status_addr[kMaxDevices] = {};
+
 }  // namespace
+
+int* fastvr::device_status_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (g_status_addr[dev] == nullptr) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_device_status) != cudaSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    g_status_addr[dev] = static_cast<int*>(ptr);
+  }
+  return g_status_addr[dev];
+}
 
 extern "C" fastvr_status_t fastvr_chunk_attn_fwd_static(
     const fastvr_attn_config_t* cfg, const void* q, int32_t q_frames,

@@ -17,6 +17,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <new>
 #include <vector>
 
@@ -51,6 +52,10 @@ struct fastvr_plan_s {
 };
 
 namespace {
+
+// Failure-detection hook for the calls without a plan (process-wide).
+std::atomic<int32_t> g_noplan_stall{0};
+std::atomic<uint64_t> g_noplan_wait_ns{0};
 
 bool valid_config(const fastvr_attn_config_t* c) {
   return c != nullptr && c->batch > 0 && c->heads > 0 && c->head_dim > 0 &&
@@ -386,7 +391,9 @@ fastvr_status_t fastvr_blockcausal_attn_fwd(const fastvr_attn_config_t* cfg,
                           ? 1.f / sqrtf((float)cfg->head_dim)
                           : cfg->softmax_scale;
   a.scale_log2 = scale * 1.4426950408889634f;
-  a.status = nullptr;
+  a.status = fastvr::device_status_word();
+  a.inject_stall = g_noplan_stall.load();
+  a.wait_limit_ns = g_noplan_wait_ns.load();
   if (fastvr::launch_blockcausal_attn(a, reinterpret_cast<cudaStream_t>(stream)) !=
       cudaSuccess)
     return FASTVR_ERR_CUDA;
@@ -463,6 +470,9 @@ fastvr_status_t fastvr_blockcausal_attn_bwd(
   a.window = cfg->window_chunks;
   a.scale = cfg->softmax_scale == 0.f ? 1.f / sqrtf((float)cfg->head_dim)
                                       : cfg->softmax_scale;
+  a.status = fastvr::device_status_word();
+  a.inject_stall = g_noplan_stall.load();
+  a.wait_limit_ns = g_noplan_wait_ns.load();
   if (fastvr::launch_blockcausal_attn_bwd(
           a, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
     return FASTVR_ERR_CUDA;
@@ -516,6 +526,26 @@ fastvr_status_t fastvr_debug_shift_next_append(fastvr_plan_t p,
 #else
   return FASTVR_ERR_UNSUPPORTED;
 #endif
+}
+
+fastvr_status_t fastvr_get_device_status(void) {
+  int* word = fastvr::device_status_word();
+  if (word == nullptr) return FASTVR_ERR_CUDA;
+  if (cudaDeviceSynchronize() != cudaSuccess) return FASTVR_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, word, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return FASTVR_ERR_CUDA;
+  if (v == fastvr::kDevOk) return FASTVR_OK;
+  const int zero = 0;
+  cudaMemcpy(word, &zero, sizeof(int), cudaMemcpyHostToDevice);
+  return v == fastvr::kDevBounds ? FASTVR_ERR_BOUNDS : FASTVR_ERR_TIMEOUT;
+}
+
+fastvr_status_t fastvr_debug_inject_stall_noplan(int32_t stall,
+                                                 uint64_t wait_limit_ns) {
+  g_noplan_stall.store(stall != 0);
+  g_noplan_wait_ns.store(wait_limit_ns);
+  return FASTVR_OK;
 }
 
 void fastvr_plan_destroy(fastvr_plan_t p) { delete p; }

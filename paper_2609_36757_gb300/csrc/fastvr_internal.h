@@ -117,7 +117,9 @@ struct OneShotParams {
   int32_t chunk_tokens;   // k * N
   int32_t window;         // W, -1 = unbounded
   float scale_log2;
-  int* status;            // control word or null (timeouts not reported)
+  int* status;            // device status word or null (not reported)
+  int32_t inject_stall;   // failure-detection test hook
+  uint64_t wait_limit_ns; // 0 = kernel default
 };
 cudaError_t launch_blockcausal_attn(const OneShotParams& p, cudaStream_t stream);
 
@@ -129,8 +131,15 @@ struct BwdArgs {
   float* scratch;  // 2 * B * H * round_up(L, 128) floats
   int32_t batch, heads, head_dim, seq_tokens, chunk_tokens, window;
   float scale;
+  int* status;             // device status word or null (not reported)
+  int32_t inject_stall;    // failure-detection test hook
+  uint64_t wait_limit_ns;  // 0 = kernel default
 };
 cudaError_t launch_blockcausal_attn_bwd(const BwdArgs& a, cudaStream_t stream);
+
+// The status word of the current device for the calls without a plan (the
+// one-shot forward and the backward), or null if it cannot be looked up.
+int* device_status_word();
 
 // Workspace parts (partial results) a launch of p uses on the current device
 // (0 when no unit is split), with at most kMaxParts parts.

@@ -74,6 +74,8 @@ SIGNATURES = {
                                             _VP]),
     "fastvr_debug_inject_stall": (_I32, [_VP, _I32, ctypes.c_uint64]),
     "fastvr_debug_shift_next_append": (_I32, [_VP, _I64]),
+    "fastvr_get_device_status": (_I32, []),
+    "fastvr_debug_inject_stall_noplan": (_I32, [_I32, ctypes.c_uint64]),
     "fastvr_plan_destroy": (None, [_VP]),
     "fastvr_status_string": (ctypes.c_char_p, [_I32]),
 }
@@ -298,6 +300,17 @@ def fastvr_debug_inject_stall(plan: int, stall: int,
 def fastvr_debug_shift_next_append(plan: int, tokens: int) -> None:
     _check(lib.fastvr_debug_shift_next_append(plan, tokens),
            "fastvr_debug_shift_next_append")
+
+
+def fastvr_get_device_status() -> int:
+    """Status of the calls without a plan on the current device (synchronises;
+    a recorded failure is cleared once returned)."""
+    return lib.fastvr_get_device_status()
+
+
+def fastvr_debug_inject_stall_noplan(stall: int, wait_limit_ns: int) -> None:
+    _check(lib.fastvr_debug_inject_stall_noplan(stall, wait_limit_ns),
+           "fastvr_debug_inject_stall_noplan")
 
 
 def fastvr_plan_destroy(plan: int) -> None:
