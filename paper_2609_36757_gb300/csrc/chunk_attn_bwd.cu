@@ -131,6 +131,18 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
   }
 }
 
+// The issuing warp's waits.  A phase that has already completed costs one
+// warp-wide try_wait and a vote (no divergent branch); otherwise lane 0
+// polls with the bounded wait and the outcome is broadcast, so the warp
+// stays converged for the elected MMA instructions.
+__device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity,
+                                              BwdShared* S) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = wait_bar(bar, parity, S);
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   const uint64_t t0 = global_timer_ns();
   while (!mbar_try_wait(bar, parity))
@@ -257,8 +269,9 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
     drain_wait(&S->full[0][i % kS0], (i / kS0) & 1);
 }
 
-// One thread issues every MMA, and a tcgen05.mma takes it about as long to
-// issue as the tensor pipe takes to run it, so the issue loops carry no
+// One warp issues every MMA (an elected lane, the warp kept converged), and
+// a tcgen05.mma takes it nearly as long to issue as the tensor pipe takes to
+// run it, so the issue loops carry no
 // descriptor arithmetic: each tile's descriptor low word is formed once per
 // call and the K steps add constant offsets (16-byte units) to it.
 
@@ -273,7 +286,7 @@ __device__ __forceinline__ void mma_nt(uint32_t sbase, uint32_t tmem, int c0,
 #pragma unroll
   for (int ks = 0; ks < D / 16; ++ks) {
     const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
-    mma_ss(tmem + c0, a_lo + off, b_lo + off, hi, kIdesc, ks > 0);
+    mma_ss_warp(tmem + c0, a_lo + off, b_lo + off, hi, kIdesc, ks > 0);
   }
 }
 
@@ -289,8 +302,8 @@ __device__ __forceinline__ void mma_tn(uint32_t sbase, uint32_t tmem, int c0,
   const uint32_t b_lo = desc_lo(sbase + b_off, kBox);
 #pragma unroll
   for (int kk = 0; kk < kT / 16; ++kk)
-    mma_ts(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
-             b_lo + (uint32_t)(kk * 2048 >> 4), hi, kIdesc, (acc | kk) != 0);
+    mma_ts_warp(tmem + c0, tmem + a0 + 64 * (kk / 4) + 8 * (kk % 4),
+                b_lo + (uint32_t)(kk * 2048 >> 4), hi, kIdesc, (acc | kk) != 0);
 }
 
 // Write 32 fp32 accumulator columns (scaled) of a TMEM row as bf16.
@@ -427,53 +440,52 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
                             p.delta + (int64_t)bh_row(p, b, h) * p.padded);
     __syncwarp();
   } else if (warp == kMmaWarp) {
-    if (lane == 0) {
-      const uint32_t sbase = smem_addr(smem);
-      // The next tile's S^T is issued right after this tile's dV (it
-      // overwrites P^T, which dV has read: the pipe runs in issue order and
-      // the compute warps keep P^T in registers), and the next dP^T right
-      // after dK (over dS^T), so the compute warps start the next tile's P
-      // as soon as they finish this tile's dS.
-      // Test hook: o_full receives no arrival before the end, so this wait
-      // runs out and exercises the abort path.
-      bool ok = (!p.inject_stall || wait_bar(&S->o_full, 0, S)) &&
-                wait_bar(&S->fixed_full, 0, S) &&
-                wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
-      if (ok) {
-        tc_fence_after();
-        mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
-        mma_commit(&S->s_ready);
-        mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
-        mma_commit(&S->dp_ready);
-      }
-      for (int j = 0; ok && j < n; ++j) {
-        const int st = j % kStages1, stn = (j + 1) % kStages1;
-        const uint32_t phn = ((j + 1) / kStages1) & 1;
-        if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
-        tc_fence_after();
-        mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
-        mma_commit(&S->empty[1][st]);  // dO_j read for the last time
-        if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[0][stn], phn, S))) break;
-          tc_fence_after();
-          mma_nt<D, L>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
-          mma_commit(&S->s_ready);
-        }
-        if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
-        tc_fence_after();
-        mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
-        mma_commit(&S->empty[0][st]);  // Q_j and the row vectors
-        if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[1][stn], phn, S))) break;
-          tc_fence_after();
-          mma_nt<D, L>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
-          mma_commit(&S->dp_ready);
-        }
-      }
-      if (ok) mma_commit(&S->o_full);
-      mma_commit(&S->drain);
-      drain_wait(&S->drain, 0);
+    const uint32_t sbase = smem_addr(smem);
+    // The next tile's S^T is issued right after this tile's dV (it
+    // overwrites P^T, which dV has read: the pipe runs in issue order and
+    // the compute warps keep P^T in registers), and the next dP^T right
+    // after dK (over dS^T), so the compute warps start the next tile's P
+    // as soon as they finish this tile's dS.
+    // Test hook: o_full receives no arrival before the end, so this wait
+    // runs out and exercises the abort path.
+    bool ok = (!p.inject_stall || wait_bar_warp(&S->o_full, 0, S)) &&
+              wait_bar_warp(&S->fixed_full, 0, S) &&
+              wait_bar_warp(&S->full[0][0], 0, S) &&
+              wait_bar_warp(&S->full[1][0], 0, S);
+    if (ok) {
+      tc_fence_after();
+      mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
+      mma_commit_warp(&S->s_ready);
+      mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
+      mma_commit_warp(&S->dp_ready);
     }
+    for (int j = 0; ok && j < n; ++j) {
+      const int st = j % kStages1, stn = (j + 1) % kStages1;
+      const uint32_t phn = ((j + 1) / kStages1) & 1;
+      if (!(ok = wait_bar_warp(&S->p_ready, j & 1, S))) break;
+      tc_fence_after();
+      mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
+      mma_commit_warp(&S->empty[1][st]);  // dO_j read for the last time
+      if (j + 1 < n) {
+        if (!(ok = wait_bar_warp(&S->full[0][stn], phn, S))) break;
+        tc_fence_after();
+        mma_nt<D, L>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
+        mma_commit_warp(&S->s_ready);
+      }
+      if (!(ok = wait_bar_warp(&S->ds_ready, j & 1, S))) break;
+      tc_fence_after();
+      mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
+      mma_commit_warp(&S->empty[0][st]);  // Q_j and the row vectors
+      if (j + 1 < n) {
+        if (!(ok = wait_bar_warp(&S->full[1][stn], phn, S))) break;
+        tc_fence_after();
+        mma_nt<D, L>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
+        mma_commit_warp(&S->dp_ready);
+      }
+    }
+    if (ok) mma_commit_warp(&S->o_full);
+    mma_commit_warp(&S->drain);
+    if (lane == 0) drain_wait(&S->drain, 0);
     __syncwarp();
   } else {
     // Compute warps: warp w owns key rows 32 (w % 4) .. + 31 (its TMEM
@@ -592,52 +604,51 @@ dq_kernel(const __grid_constant__ BwdParams p) {
                              &p.v_map, kv0, n, h, b, nullptr, nullptr);
     __syncwarp();
   } else if (warp == kMmaWarp) {
-    if (lane == 0) {
-      const uint32_t sbase = smem_addr(smem);
-      // S of the next tile is issued as soon as P of this one is in
-      // registers, so it overlaps the dS computation.
-      // Test hook: o_full receives no arrival before the end, so this wait
-      // runs out and exercises the abort path.
-      bool ok = (!p.inject_stall || wait_bar(&S->o_full, 0, S)) &&
-                wait_bar(&S->fixed_full, 0, S) &&
-                wait_bar(&S->full[0][0], 0, S) && wait_bar(&S->full[1][0], 0, S);
-      if (ok) {
-        tc_fence_after();
-        mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
-        mma_commit(&S->s_ready);
-        mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
-        mma_commit(&S->dp_ready);
-        mma_commit(&S->empty[1][0]);           // V_0 read for the last time
-      }
-      for (int j = 0; ok && j < n; ++j) {
-        // K (ring 0) and V (ring 1) run at their own depths
-        const int k_st = j % kDqS0, k_stn = (j + 1) % kDqS0;
-        const int v_stn = (j + 1) % kStages1;
-        if (!(ok = wait_bar(&S->p_ready, j & 1, S))) break;
-        if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[0][k_stn], ((j + 1) / kDqS0) & 1, S)))
-            break;
-          tc_fence_after();
-          mma_nt<D, L>(sbase, tmem, 0, 0, k_stn, 0);  // S_{j+1}
-          mma_commit(&S->s_ready);
-        }
-        if (!(ok = wait_bar(&S->ds_ready, j & 1, S))) break;
-        tc_fence_after();
-        mma_tn<D>(sbase, tmem, 256, 128, L::ring(k_st, 0, 0), j > 0);  // dQ
-        mma_commit(&S->empty[0][k_st]);  // K_j read for the last time
-        if (j + 1 < n) {
-          if (!(ok = wait_bar(&S->full[1][v_stn], ((j + 1) / kStages1) & 1, S)))
-            break;
-          tc_fence_after();
-          mma_nt<D, L>(sbase, tmem, 128, 1, v_stn, 1);  // dP_{j+1}
-          mma_commit(&S->dp_ready);
-          mma_commit(&S->empty[1][v_stn]);  // V_{j+1} read for the last time
-        }
-      }
-      if (ok) mma_commit(&S->o_full);
-      mma_commit(&S->drain);
-      drain_wait(&S->drain, 0);
+    const uint32_t sbase = smem_addr(smem);
+    // S of the next tile is issued as soon as P of this one is in
+    // registers, so it overlaps the dS computation.
+    // Test hook: o_full receives no arrival before the end, so this wait
+    // runs out and exercises the abort path.
+    bool ok = (!p.inject_stall || wait_bar_warp(&S->o_full, 0, S)) &&
+              wait_bar_warp(&S->fixed_full, 0, S) &&
+              wait_bar_warp(&S->full[0][0], 0, S) &&
+              wait_bar_warp(&S->full[1][0], 0, S);
+    if (ok) {
+      tc_fence_after();
+      mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
+      mma_commit_warp(&S->s_ready);
+      mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
+      mma_commit_warp(&S->dp_ready);
+      mma_commit_warp(&S->empty[1][0]);           // V_0 read for the last time
     }
+    for (int j = 0; ok && j < n; ++j) {
+      // K (ring 0) and V (ring 1) run at their own depths
+      const int k_st = j % kDqS0, k_stn = (j + 1) % kDqS0;
+      const int v_stn = (j + 1) % kStages1;
+      if (!(ok = wait_bar_warp(&S->p_ready, j & 1, S))) break;
+      if (j + 1 < n) {
+        if (!(ok = wait_bar_warp(&S->full[0][k_stn], ((j + 1) / kDqS0) & 1, S)))
+          break;
+        tc_fence_after();
+        mma_nt<D, L>(sbase, tmem, 0, 0, k_stn, 0);  // S_{j+1}
+        mma_commit_warp(&S->s_ready);
+      }
+      if (!(ok = wait_bar_warp(&S->ds_ready, j & 1, S))) break;
+      tc_fence_after();
+      mma_tn<D>(sbase, tmem, 256, 128, L::ring(k_st, 0, 0), j > 0);  // dQ
+      mma_commit_warp(&S->empty[0][k_st]);  // K_j read for the last time
+      if (j + 1 < n) {
+        const uint32_t v_phn = ((j + 1) / kStages1) & 1;
+        if (!(ok = wait_bar_warp(&S->full[1][v_stn], v_phn, S))) break;
+        tc_fence_after();
+        mma_nt<D, L>(sbase, tmem, 128, 1, v_stn, 1);  // dP_{j+1}
+        mma_commit_warp(&S->dp_ready);
+        mma_commit_warp(&S->empty[1][v_stn]);  // V_{j+1} read for the last time
+      }
+    }
+    if (ok) mma_commit_warp(&S->o_full);
+    mma_commit_warp(&S->drain);
+    if (lane == 0) drain_wait(&S->drain, 0);
     __syncwarp();
   } else {
     // Compute warps: warp w owns query rows 32 (w % 4) .. + 31 and key

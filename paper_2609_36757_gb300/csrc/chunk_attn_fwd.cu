@@ -278,6 +278,18 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
     drain_wait(&full[i % kStages], (i / kStages) & 1, S);
 }
 
+// The issuing warp's waits.  A phase that has already completed costs one
+// warp-wide try_wait and a vote (no divergent branch); otherwise lane 0
+// polls with the bounded wait and the outcome is broadcast, so the warp
+// stays converged for the elected MMA instructions.
+__device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity,
+                                              Shared* S, int* status) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = wait_bar(bar, parity, S, status);
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
 template <int D>
 __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
                            uint32_t tmem, const Work& w) {
@@ -288,10 +300,11 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   const int n = w.n;
   const bool two = w.nqt == 2;
 
-  // One thread issues every MMA and a tcgen05.mma takes it ~55 clk to issue
-  // against 64 clk of tensor work (M128 N128 K16), so the issue loop carries
-  // no descriptor arithmetic: the descriptor words are formed once here and
-  // each MMA only adds a constant offset (16-byte units) to the low word.
+  // One warp issues every MMA (an elected lane, the warp kept converged) and
+  // a tcgen05.mma takes it ~54 clk to issue against 64 clk of tensor work
+  // (M128 N128 K16), so the issue loop carries no descriptor arithmetic: the
+  // descriptor words are formed once here and each MMA only adds a constant
+  // offset (16-byte units) to the low word.
   const uint32_t hi = desc_hi_sw128(1024);
   const uint32_t q_lo = desc_lo(sbase + L::q(0, 0), 16);
   const uint32_t k_lo = desc_lo(sbase + L::k(0, 0), 16);
@@ -305,7 +318,7 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
       const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
-      mma_ss(tmem + t * 128, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
+      mma_ss_warp(tmem + t * 128, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
     }
   };
   // O_t += P_t V: P_t from TMEM (8 columns per 16 keys), V MN-major (d
@@ -315,24 +328,24 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     const uint32_t b0 = v_lo + (uint32_t)st * kStage16;
 #pragma unroll
     for (int kk = 0; kk < kBN / 16; ++kk)
-      mma_ts(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
+      mma_ts_warp(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
                b0 + (uint32_t)(kk * 2048 >> 4), hi, kIdescPV, (acc | kk) != 0);
   };
 
   // Test hook: o_full receives no arrival before the end of the stream, so
   // this wait runs out and exercises the abort path.
-  bool ok = !p.inject_stall || wait_bar(&S->o_full, 0, S, p.status);
-  ok = ok && wait_bar(&S->q_full, 0, S, p.status) &&
-       wait_bar(&S->k_full[0], 0, S, p.status);
+  bool ok = !p.inject_stall || wait_bar_warp(&S->o_full, 0, S, p.status);
+  ok = ok && wait_bar_warp(&S->q_full, 0, S, p.status) &&
+       wait_bar_warp(&S->k_full[0], 0, S, p.status);
   if (ok) {
     tc_fence_after();
     qk(0, 0);
-    mma_commit(&S->s_full[0]);
+    mma_commit_warp(&S->s_full[0]);
     if (two) {
       qk(1, 0);
-      mma_commit(&S->s_full[1]);
+      mma_commit_warp(&S->s_full[1]);
     }
-    mma_commit(&S->k_empty[0]);
+    mma_commit_warp(&S->k_empty[0]);
   }
   for (int j = 0; ok && j < n; ++j) {
     const int vs = j % kVStages;
@@ -340,33 +353,34 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     const int jn = j + 1;
     const int stn = jn % kKStages;
     const uint32_t phn = (jn / kKStages) & 1;
-    if (!(ok = wait_bar(&S->v_full[vs], vph, S, p.status))) break;
-    if (!(ok = wait_bar(&S->p_full[0], j & 1, S, p.status))) break;
+    if (!(ok = wait_bar_warp(&S->v_full[vs], vph, S, p.status))) break;
+    if (!(ok = wait_bar_warp(&S->p_full[0], j & 1, S, p.status))) break;
     tc_fence_after();
     pv(0, vs, j > 0);
     if (jn < n) {
-      if (!(ok = wait_bar(&S->k_full[stn], phn, S, p.status))) break;
+      if (!(ok = wait_bar_warp(&S->k_full[stn], phn, S, p.status))) break;
       tc_fence_after();
       qk(0, stn);
-      mma_commit(&S->s_full[0]);
+      mma_commit_warp(&S->s_full[0]);
     }
     if (two) {
-      if (!(ok = wait_bar(&S->p_full[1], j & 1, S, p.status))) break;
+      if (!(ok = wait_bar_warp(&S->p_full[1], j & 1, S, p.status))) break;
       tc_fence_after();
       pv(1, vs, j > 0);
     }
-    mma_commit(&S->v_empty[vs]);
+    mma_commit_warp(&S->v_empty[vs]);
     if (jn < n) {
       if (two) {
         qk(1, stn);
-        mma_commit(&S->s_full[1]);
+        mma_commit_warp(&S->s_full[1]);
       }
-      mma_commit(&S->k_empty[stn]);
+      mma_commit_warp(&S->k_empty[stn]);
     }
   }
-  if (ok) mma_commit(&S->o_full);
-  mma_commit(&S->drain);
-  drain_wait(&S->drain, 0, S);
+  if (ok) mma_commit_warp(&S->o_full);
+  mma_commit_warp(&S->drain);
+  if ((threadIdx.x & 31) == 0) drain_wait(&S->drain, 0, S);
+  __syncwarp();
 }
 
 __device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
@@ -718,8 +732,7 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     if (lane == 0) producer<D, false, kOneShot>(p, smem, S, w);
     __syncwarp();
   } else if (warp == 9) {
-    if (lane == 0) mma_issuer<D>(p, smem, S, tmem, w);
-    __syncwarp();
+    mma_issuer<D>(p, smem, S, tmem, w);
   } else {
     // A query tile that lies past the end of the chunk has no work.
     if (warp / 4 < w.nqt)
