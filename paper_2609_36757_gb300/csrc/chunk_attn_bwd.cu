@@ -131,16 +131,28 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
   }
 }
 
-// The issuing warp's waits.  A phase that has already completed costs one
-// warp-wide try_wait and a vote (no divergent branch); otherwise lane 0
-// polls with the bounded wait and the outcome is broadcast, so the warp
-// stays converged for the elected MMA instructions.
+// The issuing warp's waits: every lane polls and each decision (phase
+// complete, abort seen, time limit passed) is a warp vote, so the warp
+// never diverges and reaches the elected MMA instructions converged.  A
+// phase that has already completed costs one try_wait and one vote.
 __device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity,
                                               BwdShared* S) {
   if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
-  int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = wait_bar(bar, parity, S);
-  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+    const bool aborted = *reinterpret_cast<volatile int*>(&S->abort) != 0;
+    const bool late = global_timer_ns() - t0 > S->wait_limit_ns;
+    if (__any_sync(0xffffffffu, aborted)) return false;
+    if (__any_sync(0xffffffffu, late)) {
+      if ((threadIdx.x & 31) == 0) {
+        *reinterpret_cast<volatile int*>(&S->abort) = 1;
+        if (S->status != nullptr) atomicExch(S->status, kDevTimeout);
+      }
+      __syncwarp();
+      return false;
+    }
+  }
 }
 
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
