@@ -131,10 +131,11 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity,
   }
 }
 
-// The issuing warp's waits: every lane polls and each decision (phase
-// complete, abort seen, time limit passed) is a warp vote, so the warp
-// never diverges and reaches the elected MMA instructions converged.  A
-// phase that has already completed costs one try_wait and one vote.
+// Warp-wide waits (the MMA warp and the compute warps): every lane polls and
+// each decision (phase complete, abort seen, time limit passed) is a warp
+// vote, so the warp never diverges and reaches the elected MMA instructions
+// and the .sync.aligned TMEM loads converged.  A phase that has already
+// completed costs one try_wait and one vote.
 __device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity,
                                               BwdShared* S) {
   if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
@@ -517,7 +518,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       const int st = j % kDkdvS0;
       // the stage's LSE and D slices (the MMA warp frees the stage only after
       // ds_ready, so they stay valid while this tile is processed)
-      if (!(ok = wait_bar(&S->full[0][st], (j / kDkdvS0) & 1, S))) break;
+      if (!(ok = wait_bar_warp(&S->full[0][st], (j / kDkdvS0) & 1, S))) break;
       // -log2 LSE and -D per column
       const float* nl = reinterpret_cast<const float*>(smem + L::vec(0, st)) + 64 * hf;
       const float* nd = reinterpret_cast<const float*>(smem + L::vec(1, st)) + 64 * hf;
@@ -525,7 +526,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       float4 la[8], lb[8];
 #pragma unroll
       for (int q = 0; q < 8; ++q) la[q] = reinterpret_cast<const float4*>(nl)[q];
-      if (!(ok = wait_bar(&S->s_ready, j & 1, S))) break;
+      if (!(ok = wait_bar_warp(&S->s_ready, j & 1, S))) break;
       tc_fence_after();
       const int lo = vis_lo - i0, hi = vis_hi - i0;
       const bool need_mask = lo > 0 || hi < 64;
@@ -551,7 +552,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       // half of dP^T; the D values are read ahead like the LSE values
 #pragma unroll
       for (int q = 0; q < 8; ++q) la[q] = reinterpret_cast<const float4*>(nd)[q];
-      if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
+      if (!(ok = wait_bar_warp(&S->dp_ready, j & 1, S))) break;
       tc_fence_after();
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
@@ -568,7 +569,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->ds_ready);
     }
-    if (ok && wait_bar(&S->o_full, 0, S)) {
+    if (ok && wait_bar_warp(&S->o_full, 0, S)) {
       tc_fence_after();
       const int key = k0 + t;
       const bool in_range = key < p.seq_tokens;
@@ -687,7 +688,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     bool ok = true;
     for (int j = 0; j < n; ++j) {
       const int tok0 = kv0 + j * kT + 64 * hf;
-      if (!(ok = wait_bar(&S->s_ready, j & 1, S))) break;
+      if (!(ok = wait_bar_warp(&S->s_ready, j & 1, S))) break;
       tc_fence_after();
       const int lo = vis_lo - tok0;
       const int hi = vis_hi - tok0;
@@ -705,7 +706,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->p_ready);
       // phase 2 (overlaps the next tile's S MMAs): dS over the dP columns
-      if (!(ok = wait_bar(&S->dp_ready, j & 1, S))) break;
+      if (!(ok = wait_bar_warp(&S->dp_ready, j & 1, S))) break;
       tc_fence_after();
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
@@ -719,7 +720,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       __syncwarp();
       if (lane == 0) mbar_arrive(&S->ds_ready);
     }
-    if (ok && wait_bar(&S->o_full, 0, S)) {
+    if (ok && wait_bar_warp(&S->o_full, 0, S)) {
       tc_fence_after();
       const int64_t off = (int64_t)b * p.seq_tokens * p.heads * D +
                           (int64_t)(in_range ? row : 0) * p.heads * D +
