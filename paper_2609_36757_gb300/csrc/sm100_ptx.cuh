@@ -199,40 +199,14 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n,
          ((n >> 3) << 17) | ((m >> 4) << 24);
 }
 
-// D[tmem] (+)= A * B, issued by one thread; shared-memory operands are given
-// by their descriptor words.  mma_ss: A and B in shared memory; mma_ts: A in
-// TMEM (M rows on the lanes), B in shared memory.
-__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint32_t a_lo,
-                                         uint32_t b_lo, uint32_t hi,
-                                         uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
-      "setp.ne.b32 p, %5, 0;\n\t"
-      "mov.b64 da, {%1, %3};\n\t"
-      "mov.b64 db, {%2, %3};\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n\t}" ::"r"(
-          d_tmem),
-      "r"(a_lo), "r"(b_lo), "r"(hi), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem,
-                                         uint32_t b_lo, uint32_t hi,
-                                         uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t.reg .b64 db;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "mov.b64 db, {%2, %3};\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %5, p;\n\t}" ::"r"(
-          d_tmem),
-      "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(accumulate), "r"(idesc)
-      : "memory");
-}
-
-// The same three operations issued by a converged warp: `elect.sync` picks
-// one lane, which issues the instruction.  Every lane of the warp must reach
-// the call together.  A warp that stays converged keeps its (warp-uniform)
-// descriptor words in uniform registers: on GB300 an M128 N128 K16 MMA then
-// issues in ~54 clk instead of ~61-64 clk from a single diverged thread.
+// D[tmem] (+)= A * B issued by a converged warp: `elect.sync` picks one
+// lane, which issues the instruction, so every lane of the warp must reach
+// the call together.  Shared-memory operands are given by their descriptor
+// words.  mma_ss_warp: A and B in shared memory; mma_ts_warp: A in TMEM (M
+// rows on the lanes), B in shared memory.  A warp that stays converged keeps
+// its (warp-uniform) descriptor words in uniform registers: on GB300 an M128
+// N128 K16 MMA then issues in ~54 clk, against ~61-64 clk from one diverged
+// thread, and smaller MMAs in ~35-41 clk against ~53.
 __device__ __forceinline__ void mma_ss_warp(uint32_t d_tmem, uint32_t a_lo,
                                             uint32_t b_lo, uint32_t hi,
                                             uint32_t idesc, uint32_t accumulate) {
@@ -260,20 +234,15 @@ __device__ __forceinline__ void mma_ts_warp(uint32_t d_tmem, uint32_t a_tmem,
       "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(accumulate), "r"(idesc)
       : "memory");
 }
+
+// Arrive on `bar` once every tcgen05 op previously issued by the warp's
+// elected lane has completed (with the full warp active, `elect.sync` picks
+// the same lane as for the MMAs).
 __device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {
   asm volatile(
       "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
       "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 "
       "[%0];\n\t}" ::"r"(smem_addr(bar))
-      : "memory");
-}
-
-// Arrive on `bar` once every previously issued tcgen05 op of this thread
-// has completed.
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 "
-      "[%0];" ::"r"(smem_addr(bar))
       : "memory");
 }
 
