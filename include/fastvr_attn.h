@@ -257,7 +257,7 @@ FASTVR_API fastvr_status_t fastvr_plan_launch_count(fastvr_plan_t plan,
                                                     int64_t* launches);
 
 /* Failure-detection hook (tests).  stall != 0 makes the next attention
- * launches of this plan wait, in the MMA-issuing thread, on a barrier that
+ * launches of this plan wait, in the MMA-issuing warp, on a barrier that
  * nothing arrives on; the kernel's bounded wait runs out after
  * wait_limit_ns, every role stops, in-flight copies and MMAs are drained,
  * tensor memory is released and FASTVR_ERR_TIMEOUT is recorded for
@@ -281,7 +281,7 @@ FASTVR_API fastvr_status_t fastvr_get_device_status(void);
 
 /* Failure-detection hook (tests) for the calls without a plan, process-wide:
  * stall != 0 makes every following one-shot forward and backward launch
- * wait, in its MMA-issuing thread, on a barrier that nothing arrives on; the
+ * wait, in its MMA-issuing warp, on a barrier that nothing arrives on; the
  * bounded wait runs out after wait_limit_ns (0 = the 4 s default), every
  * role stops, in-flight copies and MMAs are drained, tensor memory is
  * released and FASTVR_ERR_TIMEOUT is recorded for fastvr_get_device_status.

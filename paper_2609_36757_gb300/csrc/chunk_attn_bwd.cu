@@ -61,7 +61,7 @@ struct BwdParams {
   int32_t seq_tokens, heads, batch, chunk_tokens, window, tiles, padded;
   float scale, scale_log2;
   int* status;             // device status word (timeouts) or null
-  int32_t inject_stall;    // test hook: the MMA thread waits on o_full first
+  int32_t inject_stall;    // test hook: the MMA warp waits on o_full first
   uint64_t wait_limit_ns;  // 0 = kWaitLimitNs
 };
 

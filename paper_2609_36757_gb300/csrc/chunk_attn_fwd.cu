@@ -12,8 +12,9 @@
 //   warp 8      TMA producer of the Q tiles (once) and the K ring (3 deep);
 //   warp 10     TMA producer of the V ring (2 deep); all tiles are
 //               128-byte swizzled boxes of 64 columns.
-//   warp 9      MMA issuer (one thread): S_t = Q_t K^T into TMEM, then
-//               O_t += P_t V with P_t read from TMEM.
+//   warp 9      MMA issuer (the warp runs converged, an elected lane
+//               issues): S_t = Q_t K^T into TMEM, then O_t += P_t V with
+//               P_t read from TMEM.
 //   warps 0-3   softmax of query tile 0, one thread per row (TMEM lane);
 //   warps 4-7   softmax of query tile 1.
 // TMEM (512 columns): S_0 | S_1 | O_0 | O_1, 128 columns each; P_t (bf16
