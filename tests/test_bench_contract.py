@@ -63,3 +63,25 @@ def test_gpu_arm_line():
     assert 2 * 8 * 3 <= d["gpu_launches"] <= 3 * 8 * 3
     c = d["clocks"]
     assert c["sm_max_mhz"] > 0 and isinstance(c["reasons"], list)
+
+
+def test_traffic_is_reported_only_for_the_profiled_source(tmp_path, monkeypatch):
+    """The roofline's `traffic` comes from a committed ncu summary only while
+    the kernel source it was taken on is unchanged (else null)."""
+    import hashlib
+    sys.path.insert(0, ROOT)
+    import bench
+    src = tmp_path / "paper_2609_36757_gb300" / "csrc" / "k.cu"
+    src.parent.mkdir(parents=True)
+    src.write_bytes(b"__global__ void k() {}\n")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    digest = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    (prof / "k_case_traffic.txt").write_text(
+        "# comment = ignored\nsource=k.cu\nsource_sha256_16=%s\n"
+        "dram_bytes_capture=10\ndram_bytes_per_avg_launch=12345\n" % digest)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.load_traffic("k_case") == 12345.0
+    assert bench.load_traffic("missing_case") is None
+    src.write_bytes(b"__global__ void k() { /* changed */ }\n")
+    assert bench.load_traffic("k_case") is None
