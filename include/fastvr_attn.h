@@ -82,7 +82,11 @@ typedef struct {
 
 typedef struct fastvr_plan_s* fastvr_plan_t;
 
-/* Bytes of device memory the caller must provide for the KV cache of cfg:
+/* Bytes of device memory the caller must provide for the KV cache of cfg.
+ * The cache is the one of streaming inference (Sec. 3.1, last paragraph):
+ * it keeps the keys and values of the chunks that later queries still see
+ * under Eq. 1 with window W, so it holds O(k) tokens per head for a bounded
+ * window.  Layout:
  * K and V, each [B, H, S*k*N, d] bfloat16 with S = window_chunks + 1 slots
  * (bounded window) or max_chunks slots (unbounded), then the attention
  * kernel's split-KV workspace (256 x 256 x (d + 1) floats), then a 256-byte
@@ -92,7 +96,10 @@ FASTVR_API fastvr_status_t fastvr_kv_cache_bytes(const fastvr_attn_config_t* cfg
                                       size_t* bytes);
 
 /* Validate cfg and bind a caller-owned cache buffer of `bytes` bytes (device
- * memory, 256-byte aligned, at least fastvr_kv_cache_bytes).  The cache
+ * memory, 256-byte aligned, at least fastvr_kv_cache_bytes).  The plan holds
+ * the streaming state of Sec. 3.1 (last paragraph): the chunk counter c and
+ * the ring of cache slots, from which each chunk's visible set under Eq. 1
+ * (chunks max(0, c-W) .. c) is resolved on the host.  The cache
  * contents need no initialisation.  Host only: device set-up (TMA
  * descriptors, device check, clearing the control block) happens on the
  * first device call.  *out receives a new plan, released by
@@ -235,11 +242,13 @@ FASTVR_API fastvr_status_t fastvr_one_step_update(const void* z_lq,
  * kernels, same work split).  The first call on each device resolves the
  * array's device address (a symbol lookup, no allocation): make that first
  * call before any stream capture.  Every call on a device shares the array
- * and it keeps the last call's contents (each call clears the status word
- * first), so calls that overlap on the GPU (other streams, other threads)
- * race: serialise them.  A bounded-wait timeout leaves out undefined and is
- * not reported.  No cudaMalloc, cudaFree or allocating library routine is
- * called.
+ * and it keeps the last call's contents (nothing in it needs clearing:
+ * every partial result is written before it is read), so calls that overlap
+ * on the GPU (other streams, other threads) race: serialise them.  A bounded-wait timeout leaves out undefined and is
+ * recorded in the per-device status word that fastvr_get_device_status
+ * reports.  No cudaMalloc, cudaFree or allocating library routine is
+ * called.  Limits: q_frames * N and every seg_start + seg_len at most
+ * 2^30 - 1 (the kernels index tokens in 32 bits); softmax_scale finite.
  * Errors: INVALID_ARG (null or misaligned pointers, bad sizes or ranges),
  * UNSUPPORTED (head_dim, device not sm_103), CAPACITY (the call's split
  * needs more partial results than the array holds: 190 at d = 128, 378 at
@@ -270,7 +279,8 @@ FASTVR_API fastvr_status_t fastvr_debug_inject_stall(fastvr_plan_t plan,
                                                      uint64_t wait_limit_ns);
 
 /* Device-side failures of the calls without a plan (the one-shot forward
- * fastvr_blockcausal_attn_fwd and the backward fastvr_blockcausal_attn_bwd):
+ * fastvr_blockcausal_attn_fwd, the backward fastvr_blockcausal_attn_bwd and
+ * the allocation-free fastvr_chunk_attn_fwd_static):
  * a bounded wait that gave up — or, in the debug library, a failed index
  * check — is recorded in a status word of the current device, shared by all
  * such calls on it.  This call waits for the device to finish (it

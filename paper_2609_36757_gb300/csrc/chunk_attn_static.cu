@@ -10,10 +10,12 @@
 // workspace region that the plan's cache buffer carries.
 //
 // The split-KV scratch (partial results of the units that are cut along the
-// keys) and the status word live instead in one file-scope device array of a
-// fixed size, which every GPU that loads this library holds until exit.  The
-// kernels are the ones fastvr_chunk_attn_fwd launches, with the same work
-// split, so the outputs are the same.
+// keys) lives instead in one file-scope device array of a fixed size, which
+// every GPU that loads this library holds until exit.  The kernels are the
+// ones fastvr_chunk_attn_fwd launches, with the same work split, so the
+// outputs are the same.  A bounded wait that gives up is recorded in the
+// per-device status word of the calls without a plan (also a file-scope
+// device variable), which fastvr_get_device_status reads and clears.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -26,10 +28,9 @@
 
 namespace {
 
-// 24 MiB: room for the status word and 190 partial results at d = 128
-// (378 at d = 64); a GB300 launch uses at most one per SM (152).
+// 24 MiB: room for 190 partial results at d = 128 (378 at d = 64); a GB300
+// launch uses at most one per SM (152).
 constexpr size_t kScratchBytes = size_t(24) << 20;
-constexpr size_t kStatusBytes = 256;
 
 static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
@@ -89,13 +90,21 @@ extern "C" fastvr_status_t fastvr_chunk_attn_fwd_static(
       seg_len == nullptr || q_frames < 1 || cache_tokens < 1 ||
       num_segments < 1 || num_segments > fastvr::kMaxSegments ||
       cfg->batch < 1 || cfg->heads < 1 || cfg->tokens_per_frame < 1 ||
-      !(cfg->softmax_scale >= 0.f) || !aligned16(q) || !aligned16(out) ||
+      !(cfg->softmax_scale >= 0.f) || !isfinite(cfg->softmax_scale) ||
+      !aligned16(q) || !aligned16(out) ||
       !aligned16(k_cache) || !aligned16(v_cache) || (((uintptr_t)lse) & 3u))
     return FASTVR_ERR_INVALID_ARG;
   if (cfg->head_dim != 64 && cfg->head_dim != 128) return FASTVR_ERR_UNSUPPORTED;
+  // The kernels index query rows and key tokens in 32-bit arithmetic (a key
+  // coordinate is a segment start plus a tile offset), so the query length
+  // and the end of every segment must stay within INT32_MAX / 2.
+  const int64_t q_tokens = (int64_t)q_frames * cfg->tokens_per_frame;
+  if (q_tokens > INT32_MAX / 2) return FASTVR_ERR_INVALID_ARG;
   for (int s = 0; s < num_segments; ++s)
-    if (seg_start[s] < 0 || seg_len[s] < 1 || seg_len[s] > INT32_MAX ||
-        seg_start[s] > INT32_MAX || seg_start[s] + seg_len[s] > cache_tokens)
+    if (seg_start[s] < 0 || seg_len[s] < 1 || seg_len[s] > INT32_MAX / 2 ||
+        seg_start[s] > INT32_MAX / 2 ||
+        seg_start[s] + seg_len[s] > INT32_MAX / 2 ||
+        seg_start[s] + seg_len[s] > cache_tokens)
       return FASTVR_ERR_INVALID_ARG;
 
   int dev = 0, major = 0, minor = 0;
@@ -120,7 +129,7 @@ extern "C" fastvr_status_t fastvr_chunk_attn_fwd_static(
   a.batch = cfg->batch;
   a.heads = cfg->heads;
   a.head_dim = d;
-  a.q_tokens = q_frames * cfg->tokens_per_frame;
+  a.q_tokens = (int32_t)q_tokens;
   a.q_str.head = d;
   a.q_str.token = (int64_t)cfg->heads * d;
   a.q_str.batch = (int64_t)a.q_tokens * cfg->heads * d;
@@ -137,20 +146,20 @@ extern "C" fastvr_status_t fastvr_chunk_attn_fwd_static(
       cfg->softmax_scale == 0.f ? 1.f / sqrtf((float)d) : cfg->softmax_scale;
   a.scale_log2 = scale * 1.4426950408889634f;
 
-  // Scratch layout: partial results, then the status word in the last
-  // kStatusBytes.  A call whose split needs more partial results than fit
-  // is refused rather than run with a different split.
+  // The array holds partial results only.  A call whose split needs more of
+  // them than fit is refused rather than run with a different split.  The
+  // array keeps the last call's contents, which needs no clearing: every
+  // partial result is written before it is read.
   const size_t part_bytes = (size_t)fastvr::kUnitRows * (d + 1) * sizeof(float);
-  const int capacity = (int)((kScratchBytes - kStatusBytes) / part_bytes);
+  const int capacity = (int)(kScratchBytes / part_bytes);
   if (fastvr::chunk_attn_parts(a) > capacity) return FASTVR_ERR_CAPACITY;
   a.workspace = reinterpret_cast<float*>(scratch);
   a.workspace_parts = capacity;
-  a.status = reinterpret_cast<int*>(scratch + kScratchBytes - kStatusBytes);
-  // The array keeps the last call's contents: the status word must start at
-  // zero (partial results are always written before they are read).
+  // Timeouts go to the sticky per-device word (zero at load, cleared when
+  // fastvr_get_device_status reads it).
+  a.status = fastvr::device_status_word();
+  if (a.status == nullptr) return FASTVR_ERR_CUDA;
   const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(a.status, 0, sizeof(int), st) != cudaSuccess)
-    return FASTVR_ERR_CUDA;
   int launched = 0;
   if (fastvr::launch_chunk_attn(a, st, &launched) != cudaSuccess)
     return FASTVR_ERR_CUDA;

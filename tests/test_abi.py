@@ -249,16 +249,26 @@ def test_static_entry_rejects_bad_arguments_before_any_device_work(fv):
         dict(q=0), dict(q_frames=0), dict(cache_tokens=0),
         dict(segments=[(0, 64)] * 3), dict(segments=[(0, 0)]),
         dict(segments=[(200, 100)]), dict(segments=[(-1, 10)]),
-        dict(q=FAKE + 8), dict(out=FAKE + 4),
+        dict(q=FAKE + 8), dict(out=FAKE + 4), dict(k=FAKE + 2),
+        dict(v=FAKE + 8), dict(lse=FAKE + 2),
+        # q_frames * N past 2^30 - 1 (32-bit token indexing in the kernels)
+        dict(q_frames=1 << 24),
+        # a segment ending past 2^30 - 1, even inside a huge cache
+        dict(segments=[((1 << 30) - 64, 128)], cache_tokens=1 << 40),
+        dict(segments=[(0, 128), ((1 << 31), 128)], cache_tokens=1 << 40),
+        dict(cfg=fv.make_config(1, 2, 128, 64, 2, -1, 4, float("inf"))),
+        dict(cfg=fv.make_config(1, 2, 128, 64, 2, -1, 4, float("nan"))),
+        dict(cfg=fv.make_config(1, 2, 128, 64, 2, -1, 4, -1.0)),
     ]
     for kw in cases:
-        a = dict(q=FAKE, q_frames=1, k=FAKE, v=FAKE, cache_tokens=256,
-                 segments=ok_seg, out=FAKE)
+        a = dict(cfg=cfg, q=FAKE, q_frames=1, k=FAKE, v=FAKE,
+                 cache_tokens=256, segments=ok_seg, out=FAKE, lse=0)
         a.update(kw)
         with pytest.raises(fv.FastVRError) as e:
-            fv.fastvr_chunk_attn_fwd_static(cfg, a["q"], a["q_frames"], a["k"],
-                                            a["v"], a["cache_tokens"],
-                                            a["segments"], a["out"], 0, 0)
+            fv.fastvr_chunk_attn_fwd_static(a["cfg"], a["q"], a["q_frames"],
+                                            a["k"], a["v"], a["cache_tokens"],
+                                            a["segments"], a["out"], a["lse"],
+                                            0)
         assert e.value.status == fv.FASTVR_ERR_INVALID_ARG, kw
     bad_d = fv.make_config(1, 2, 96, 64, 2, -1, 4)
     with pytest.raises(fv.FastVRError) as e:

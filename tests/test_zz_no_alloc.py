@@ -7,8 +7,11 @@ split-KV scratch is a fixed device array inside the library instead of the
 workspace region of a plan's cache buffer.  Here it is called through the C
 ABI, twice in a row per chunk, on K/V that live in a plan's cache, and each
 output must match the plan entry point's output on the same inputs within
-the tolerances the parity tests use.  The file is collected last so that a
-run that stops at its first failure has already run every other test."""
+the tolerances the parity tests use.  The device's free memory must not move
+across a call, some chunk of each case must be split along the keys (so the
+static scratch is really used), and no timeout may be recorded.  The file is
+collected last so that a run that stops at its first failure has already run
+every other test."""
 import pytest
 import torch
 
@@ -45,20 +48,31 @@ def test_static_scratch_entry_matches_plan_entry_on_two_calls(w):
     k_ptr = att.cache.data_ptr()
     v_ptr = k_ptr + _region_bytes(w, slots)
     stream = torch.cuda.current_stream().cuda_stream
+    splits = 0
     for c, q, k, v in WL.chunk_stream(w):
         att.append(k.cuda(), v.cuda())
         qd = q.cuda()
+        before = att.launch_count()
         ref_o, ref_l = att.forward(qd, want_lse=True)
+        # two launches: some units were cut along the keys, so the partial
+        # results went through the scratch (the same split in both paths)
+        splits += att.launch_count() - before == 2
         segments, _ = att.visible()
         frames = q.shape[1] // w.tokens_per_frame
         prev = None
         for call in range(2):
             o = torch.full_like(qd, float("nan"))
             lse = torch.full_like(ref_l, float("nan"))
+            torch.cuda.synchronize()
+            free_before = torch.cuda.mem_get_info()[0]
             FV.fastvr_chunk_attn_fwd_static(
                 cfg, qd.data_ptr(), frames, k_ptr, v_ptr, cache_tokens,
                 segments, o.data_ptr(), lse.data_ptr(), stream)
             torch.cuda.synchronize()
+            if call == 1:
+                # the device's free memory is unchanged by a call (the first
+                # call on a device may load the library's kernels)
+                assert torch.cuda.mem_get_info()[0] == free_before
             err = Err()
             err.add(to64(o.cpu()), to64(ref_o.cpu()), lse.cpu().numpy(),
                     ref_l.cpu().double().numpy())
@@ -67,3 +81,6 @@ def test_static_scratch_entry_matches_plan_entry_on_two_calls(w):
                 assert torch.equal(o, prev), f"calls differ at chunk {c}"
             prev = o
     assert att.status() == FV.FASTVR_OK
+    assert FV.fastvr_get_device_status() == FV.FASTVR_OK
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert splits > 0, f"no chunk of {w.name} was split on {sms} SMs"
