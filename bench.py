@@ -72,9 +72,10 @@ def load_peaks():
             "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def load_traffic(kernel: str):
-    """DRAM bytes per launch from a committed ncu summary, when that summary
-    was taken on the current kernel source (else None)."""
+def load_profile(kernel: str):
+    """The key=value lines of a committed ncu summary
+    (profiles/<kernel>_traffic.txt), when that summary was taken on the
+    current kernel source (else None)."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
     if not os.path.exists(path):
@@ -90,7 +91,31 @@ def load_traffic(kernel: str):
     digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     if digest != kv.get("source_sha256_16"):
         return None
-    return float(kv["dram_bytes_per_avg_launch"])
+    return kv
+
+
+def load_traffic(kernel: str):
+    """DRAM bytes per average launch from a committed ncu summary taken on
+    the current kernel source (else None)."""
+    kv = load_profile(kernel)
+    return None if kv is None else float(kv["dram_bytes_per_avg_launch"])
+
+
+def append_dram(peaks):
+    """What DRAM saw during one 1080p kv_append launch (ncu), beside the
+    event-timed rate that counts every byte the append reads and writes."""
+    kv = load_profile("kv_append_1080p")
+    if kv is None:
+        return None
+    rd = float(kv["dram_read_bytes"])
+    wr = float(kv["dram_write_bytes_during_launch"])
+    t = float(kv["ncu_time_ns"]) * 1e-9
+    return {"read_bytes": rd, "write_bytes_during_launch": wr,
+            "algorithmic_bytes": float(kv["algorithmic_read_bytes"]) +
+            float(kv["algorithmic_write_bytes"]),
+            "ncu_us": t * 1e6, "dram_gbs_during_launch": (rd + wr) / t / 1e9,
+            "dram_frac_of_hbm": (rd + wr) / t / 1e9 / peaks["hbm_gbs"],
+            "source": "profiles/kv_append_1080p_traffic.txt (ncu)"}
 
 
 # ------------------------------------------------------------- clocks
@@ -238,61 +263,24 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
     dq = [q.to(dev) for q, _, _ in chunks]
     dk = [k.to(dev) for _, k, _ in chunks]
     dv = [v.to(dev) for _, _, v in chunks]
-    douts = [torch.empty_like(q) for q in dq]
     att = FV.StreamingAttention(FV.config_from_workload(w), dev)
-    stream = torch.cuda.current_stream(dev)
-
-    def step(ev=None):
-        att.reset()
-        for c in range(w.num_chunks):
-            if ev is not None:
-                ev[c][0].record(stream)
-            att.append(dk[c], dv[c])
-            if ev is not None:
-                ev[c][1].record(stream)
-            att.forward(dq[c], out=douts[c])
-            if ev is not None:
-                ev[c][2].record(stream)
-
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize(dev)
-    if att.status() != FV.FASTVR_OK:
-        raise RuntimeError("device-side failure during warm-up")
-
-    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)]
-            for _ in range(w.num_chunks)] for _ in range(args.steps)]
-    clocks = ClockSampler(local_rank) if rank == 0 else None
-    if clocks:
-        clocks.start()
-        time.sleep(0.3)
-    barrier(world)
-    torch.cuda.synchronize(dev)
-    launches_before = att.launch_count()
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
-    t_start.record(stream)
-    for s in range(args.steps):
-        step(evs[s])
-    t_end.record(stream)
-    launches = att.launch_count() - launches_before
-    torch.cuda.synchronize(dev)
-    barrier(world)
-    clock_info = clocks.stop() if clocks else None
-    elapsed_ms = t_start.elapsed_time(t_end)
-    if att.status() != FV.FASTVR_OK:
-        raise RuntimeError("device-side failure in the timed region")
-
-    fwd_ms = [[evs[s][c][1].elapsed_time(evs[s][c][2]) for c in range(w.num_chunks)]
-              for s in range(args.steps)]
-    app_ms = [[evs[s][c][0].elapsed_time(evs[s][c][1]) for c in range(w.num_chunks)]
-              for s in range(args.steps)]
-    max_ms = reduce_max(elapsed_ms, world)
+    t = time_stream(att, w, dq, dk, dv, args.steps, args.warmup, dev,
+                    local_rank if rank == 0 else None, world)
+    fwd_ms, app_ms, launches = t["fwd_ms"], t["app_ms"], t["launches"]
+    clock_info = t["clocks"]
+    max_ms = reduce_max(t["elapsed_ms"], world)
     value = world * step_flops * args.steps / (max_ms / 1e3) / 1e12
 
     e2e = (None if args.skip_e2e else
            run_e2e(args, w, chunks, att, dev, step_flops, world))
     one_step = measure_one_step(dev)
+    del dq, dk, dv, att
+    per_workload = None
+    if args.per_workload and world == 1:
+        peaks, _ = load_peaks()
+        per_workload = {name: measure_workload(WL.WORKLOADS[name], dev,
+                                               peaks, local_rank)
+                        for name in PER_WORKLOADS}
 
     if rank != 0:
         return
@@ -339,6 +327,7 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
         "frac_of_burst_peak": attn_tflops / peaks["bf16_tflops"],
         "append_gbs": app_gbs,
         "append_frac_of_hbm": app_gbs / peaks["hbm_gbs"],
+        "append_dram": append_dram(peaks) if w.name == "1080p" else None,
         "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peak,
                      "unit": "TFLOP/s", "frac": attn_tflops / peak,
                      "peak_kind": f"{peak_kind} bf16 sustained",
@@ -350,12 +339,119 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
         "clocks": clock_info,
         "e2e": e2e,
     }
+    if per_workload is not None:
+        line["per_workload"] = per_workload
     if world == 1 and args.cpu_seconds > 0:
         cpu_v, desc = OracleSample(w, chunks).run(args.cpu_seconds, 10 ** 6)
         line["cpu_baseline"] = {"value": cpu_v, "unit": UNIT,
                                 "cores": HOST_CORES, "kind": "oracle",
                                 "sample": desc}
     print(json.dumps(line), flush=True)
+
+
+def time_stream(att, w, dq, dk, dv, steps, warmup, dev, clock_index, world):
+    """Stream w's chunks (device tensors dq/dk/dv) through `att`: `warmup`
+    untimed steps, then `steps` timed ones, each reset + per chunk (append,
+    forward), with CUDA events on the launching stream around every launch
+    and around the whole timed region (bracketed by a barrier and device
+    synchronisation).  Clocks are sampled during the timed region when
+    clock_index is a device index."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    douts = [torch.empty_like(q) for q in dq]
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        att.reset()
+        for c in range(w.num_chunks):
+            if ev is not None:
+                ev[c][0].record(stream)
+            att.append(dk[c], dv[c])
+            if ev is not None:
+                ev[c][1].record(stream)
+            att.forward(dq[c], out=douts[c])
+            if ev is not None:
+                ev[c][2].record(stream)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    if att.status() != FV.FASTVR_OK:
+        raise RuntimeError("device-side failure during warm-up")
+
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            for _ in range(w.num_chunks)] for _ in range(steps)]
+    clocks = ClockSampler(clock_index) if clock_index is not None else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    launches_before = att.launch_count()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for s in range(steps):
+        step(evs[s])
+    t_end.record(stream)
+    launches = att.launch_count() - launches_before
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clock_info = clocks.stop() if clocks else None
+    if att.status() != FV.FASTVR_OK:
+        raise RuntimeError("device-side failure in the timed region")
+    return {
+        "elapsed_ms": t_start.elapsed_time(t_end),
+        "fwd_ms": [[evs[s][c][1].elapsed_time(evs[s][c][2])
+                    for c in range(w.num_chunks)] for s in range(steps)],
+        "app_ms": [[evs[s][c][0].elapsed_time(evs[s][c][1])
+                    for c in range(w.num_chunks)] for s in range(steps)],
+        "launches": launches, "clocks": clock_info,
+    }
+
+
+# The other streams of the metric (480p, 720p peaked, windowed 1080p) and the
+# paper's own inference shape (k = 3, W = 1, six 64 x 64 latent tiles on B).
+PER_WORKLOADS = ("480p", "720p-peaked", "1080p-windowed", "paper-tiles-64x64")
+
+
+def measure_workload(w, dev, peaks, clock_index, steps: int = 3,
+                     warmup: int = 3):
+    """One stream's numbers with the headline's method: inputs drawn on the
+    device with the workload's recipe (resident in HBM), path TFLOP/s over
+    the whole timed region, kernel TFLOP/s over the attention launches'
+    events, per-chunk ms, latent frames/s, and the clocks of this leg."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    lk = visible_tokens_per_chunk(w)
+    flops = [chunk_flops(w, lk[c], c) for c in range(w.num_chunks)]
+    data = [(q, k, v) for _, q, k, v in WL.chunk_stream(w, device=str(dev))]
+    dq, dk, dv = ([x[i] for x in data] for i in range(3))
+    att = FV.StreamingAttention(FV.config_from_workload(w), dev)
+    t = time_stream(att, w, dq, dk, dv, steps, warmup, dev, clock_index, 1)
+    del data, dq, dk, dv, att
+    torch.cuda.empty_cache()
+    path = sum(flops) * steps / (t["elapsed_ms"] / 1e3) / 1e12
+    kernel = sum(flops) * steps / (sum(map(sum, t["fwd_ms"])) / 1e3) / 1e12
+    per_chunk = [statistics.median(t["fwd_ms"][s][c] for s in range(steps))
+                 for c in range(w.num_chunks)]
+    return {
+        "steps": steps, "warmup": warmup,
+        "shape": {"batch": w.batch, "heads": w.heads, "head_dim": w.head_dim,
+                  "tokens_per_frame": w.tokens_per_frame,
+                  "frames_per_chunk": w.frames_per_chunk,
+                  "chunks": w.num_chunks, "window_chunks": w.window_chunks,
+                  "last_chunk_frames": w.last_chunk_frames or
+                  w.frames_per_chunk, "peaked": w.peaked},
+        "flops_per_step": sum(flops),
+        "path_tflops": path, "kernel_tflops": kernel,
+        "ms_per_chunk": {"mean_fwd": statistics.mean(per_chunk),
+                         "last_fwd": per_chunk[-1],
+                         "mean_step_per_chunk": t["elapsed_ms"] / steps /
+                         w.num_chunks},
+        "latent_frames_per_s": w.num_frames * steps / (t["elapsed_ms"] / 1e3),
+        "kernel_frac_of_sustained": kernel / peaks["bf16_tflops_sustained"],
+        "kernel_frac_of_burst": kernel / peaks["bf16_tflops"],
+        "gpu_launches": t["launches"], "clocks": t["clocks"],
+    }
 
 
 def measure_one_step(dev, sets: int = 8, rounds: int = 3):
@@ -559,6 +655,11 @@ def main(argv=None):
                          "forward + backward (extra measurements)")
     ap.add_argument("--skip-e2e", action="store_true",
                     help="omit the end-to-end leg (profiling cases)")
+    ap.add_argument("--no-per-workload", dest="per_workload",
+                    action="store_false",
+                    help="omit the per-workload legs (480p, 720p peaked, "
+                         "windowed 1080p, paper tiles) run after the "
+                         "headline at N = 1")
     args = ap.parse_args(argv)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -99,19 +99,25 @@ WORKLOADS = {w.name: w for w in
               PAPER_TILES_32, PAPER_TILES_64, TRAIN_CLIP)}
 
 
-def chunk_stream(w: Workload) -> Iterator[Tuple[int, torch.Tensor, torch.Tensor,
-                                                torch.Tensor]]:
-    """Yield (c, Q_c, K_c, V_c) as bfloat16 CPU tensors [B, f_c*N, H, d]."""
-    g = torch.Generator(device="cpu")
+def chunk_stream(w: Workload, device: str = "cpu"
+                 ) -> Iterator[Tuple[int, torch.Tensor, torch.Tensor,
+                                 torch.Tensor]]:
+    """Yield (c, Q_c, K_c, V_c) as bfloat16 tensors [B, f_c*N, H, d].
+
+    With the default CPU device these are the seeded inputs that the CUDA
+    path and the oracle share.  Another device draws with the same recipe
+    from that device's generator (other values: for timing only)."""
+    g = torch.Generator(device=device)
     g.manual_seed(w.seed)
     for c in range(w.num_chunks):
         shape = w.chunk_shape(c)
-        q = torch.randn(shape, generator=g, dtype=torch.float32)
-        k = torch.randn(shape, generator=g, dtype=torch.float32)
-        v = torch.randn(shape, generator=g, dtype=torch.float32)
+        kw = dict(generator=g, dtype=torch.float32, device=device)
+        q = torch.randn(shape, **kw)
+        k = torch.randn(shape, **kw)
+        v = torch.randn(shape, **kw)
         if w.peaked:
-            uq = torch.rand(shape[:2], generator=g, dtype=torch.float32)
-            uk = torch.rand(shape[:2], generator=g, dtype=torch.float32)
+            uq = torch.rand(shape[:2], **kw)
+            uk = torch.rand(shape[:2], **kw)
             q = q * (0.5 + 1.5 * uq)[:, :, None, None]
             k = k * (0.5 + 1.5 * uk)[:, :, None, None]
         yield (c, q.to(torch.bfloat16), k.to(torch.bfloat16),

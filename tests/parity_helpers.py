@@ -10,6 +10,7 @@ import numpy as np
 import torch
 
 from oracle import attention as OA
+import oracle_pool
 from paper_2609_36757_gb300 import workloads as WL
 
 # Tolerances on the attention output (bf16 in, fp32 accumulate, bf16 out):
@@ -87,20 +88,30 @@ def to64(t: torch.Tensor) -> np.ndarray:
     return t.float().numpy().astype(np.float64)
 
 
+def bf16_bits(t: torch.Tensor) -> np.ndarray:
+    """The 16-bit patterns of a bfloat16 CPU tensor (contiguous copy)."""
+    return t.contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
 def run_stream(w: WL.Workload, rows_per_chunk: Optional[int] = None,
                heads: Optional[List[int]] = None, chunk_stride: int = 1,
                device: str = "cuda") -> Err:
     """Stream every chunk of `w` through the library (append then forward).
 
     rows_per_chunk None compares every output element; otherwise the oracle
-    computes exact values for sampled rows only (rows are independent).  Only
-    every `chunk_stride`-th chunk (and the last) is compared, all heads unless
-    `heads` is given."""
+    computes exact values for sampled rows only (rows are independent), one
+    (chunk, batch, head) per worker process of `oracle_pool`, while the GPU
+    streams on.  Only every `chunk_stride`-th chunk (and the last) is
+    compared, all heads unless `heads` is given."""
     from paper_2609_36757_gb300 import fastvr as FV
     att = FV.StreamingAttention(FV.config_from_workload(w), device)
     window = collections.deque()  # (c, k, v) of chunks still visible
     err = Err()
     scale = w.softmax_scale
+    pend = None
+    if rows_per_chunk is not None:
+        pend = oracle_pool.Pending(
+            lambda got, ref: err.add(got[0], ref[0], got[1], ref[1]))
     for c, q, k, v in WL.chunk_stream(w):
         att.append(k.to(device), v.to(device))
         o, lse = att.forward(q.to(device), want_lse=True)
@@ -116,6 +127,16 @@ def run_stream(w: WL.Workload, rows_per_chunk: Optional[int] = None,
         rows = (np.arange(Lq) if rows_per_chunk is None else
                 sample_rows(Lq, w.tokens_per_frame, rows_per_chunk, 1000 + c))
         hs = range(w.heads) if heads is None else heads
+        if pend is not None:
+            for b in range(w.batch):
+                for h in hs:
+                    task = (bf16_bits(q[b, rows, h]),
+                            bf16_bits(torch.cat([e[1][b, :, h] for e in window])),
+                            bf16_bits(torch.cat([e[2][b, :, h] for e in window])),
+                            scale)
+                    pend.submit((to64(o[b, rows, h]), lse[b, h, rows].numpy()),
+                                task)
+            continue
         kvis = torch.cat([e[1] for e in window], dim=1)
         vvis = torch.cat([e[2] for e in window], dim=1)
         for b in range(w.batch):
@@ -125,5 +146,7 @@ def run_stream(w: WL.Workload, rows_per_chunk: Optional[int] = None,
                     to64(vvis[b, :, h]), scale)
                 err.add(to64(o[b, rows, h]), ref_o,
                         lse[b, h, rows].numpy(), ref_l)
+    if pend is not None:
+        pend.finish()
     assert att.status() == FV.FASTVR_OK
     return err
