@@ -55,6 +55,11 @@ constexpr int kVStages = 2;     // depth of the V ring
 constexpr int kThreads = 352;   // 8 softmax warps, K and V producers, MMA
 constexpr int kBox = 128 * 128; // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr uint32_t kTmemCols = 512;
+// TMEM columns: one S tile shared by the two query tiles, P_0 and P_1 (bf16
+// pairs, 64 columns each), O_0 and O_1.
+constexpr uint32_t kTmemS = 0;
+constexpr uint32_t kTmemP = 128;
+constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleThreshold = 8.0f;      // log2 units
 constexpr int kMinTilesPerPart = 4;             // key tiles per split part
 constexpr uint64_t kDefaultWaitLimitNs = 4000000000ull;  // 4 s per wait
@@ -160,7 +165,8 @@ struct Shared {
   uint64_t q_full;
   uint64_t k_full[kKStages], k_empty[kKStages];
   uint64_t v_full[kVStages], v_empty[kVStages];
-  uint64_t s_full[kQTiles], p_full[kQTiles];
+  uint64_t s_full[kQTiles], p_full[kQTiles], p_free[kQTiles];
+  uint64_t s_free;
   uint64_t o_full, drain;
   uint32_t tmem_base;
   int abort;
@@ -323,71 +329,86 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   const uint32_t k_lo = desc_lo(sbase + L::k(0, 0), 16);
   const uint32_t v_lo = desc_lo(sbase + L::v(0, 0), kBox);
   constexpr uint32_t kStage16 = (uint32_t)(L::kNB * kBox) >> 4;
-  // S_t = Q_t K^T: both operands K-major, 128-byte swizzle; a K step of 16
-  // elements is 32 bytes inside a 64-column box.
+  // S = Q_t K^T into the shared S columns: both operands K-major, 128-byte
+  // swizzle; a K step of 16 elements is 32 bytes inside a 64-column box.
   auto qk = [&](int t, int st) {
     const uint32_t a0 = q_lo + (uint32_t)(L::q(t, 0) >> 4);
     const uint32_t b0 = k_lo + (uint32_t)st * kStage16;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
       const uint32_t off = (uint32_t)((ks / 4) * kBox + (ks % 4) * 32) >> 4;
-      mma_ss_warp(tmem + t * 128, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
+      mma_ss_warp(tmem + kTmemS, a0 + off, b0 + off, hi, kIdescQK, ks > 0);
     }
   };
-  // O_t += P_t V: P_t from TMEM (8 columns per 16 keys), V MN-major (d
+  // O_t += P_t V: P_t from its TMEM columns (8 per 16 keys), V MN-major (d
   // contiguous): 16 keys are two 8-row groups (2048 bytes), the two 64-column
   // halves of d are one box apart.
   auto pv = [&](int t, int st, int acc) {
     const uint32_t b0 = v_lo + (uint32_t)st * kStage16;
 #pragma unroll
     for (int kk = 0; kk < kBN / 16; ++kk)
-      mma_ts_warp(tmem + 256 + t * 128, tmem + t * 128 + kk * 8,
-               b0 + (uint32_t)(kk * 2048 >> 4), hi, kIdescPV, (acc | kk) != 0);
+      mma_ts_warp(tmem + kTmemO + t * 128, tmem + kTmemP + t * 64 + kk * 8,
+                  b0 + (uint32_t)(kk * 2048 >> 4), hi, kIdescPV,
+                  (acc | kk) != 0);
+  };
+  // The k-th QK^T (of either tile) may overwrite S once the softmax warps
+  // have read the previous one into registers (completion k - 1 of s_free).
+  int s_uses = 0;
+  auto take_s = [&]() -> bool {
+    if (s_uses > 0 &&
+        !wait_bar_warp(&S->s_free, (uint32_t)(s_uses - 1) & 1, S, p.status))
+      return false;
+    ++s_uses;
+    tc_fence_after();
+    return true;
   };
 
   // Test hook: o_full receives no arrival before the end of the stream, so
   // this wait runs out and exercises the abort path.
   bool ok = !p.inject_stall || wait_bar_warp(&S->o_full, 0, S, p.status);
-  ok = ok && wait_bar_warp(&S->q_full, 0, S, p.status) &&
-       wait_bar_warp(&S->k_full[0], 0, S, p.status);
-  if (ok) {
-    tc_fence_after();
-    qk(0, 0);
-    mma_commit_warp(&S->s_full[0]);
-    if (two) {
-      qk(1, 0);
-      mma_commit_warp(&S->s_full[1]);
-    }
-    mma_commit_warp(&S->k_empty[0]);
-  }
-  for (int j = 0; ok && j < n; ++j) {
-    const int vs = j % kVStages;
-    const uint32_t vph = (j / kVStages) & 1;
-    const int jn = j + 1;
-    const int stn = jn % kKStages;
-    const uint32_t phn = (jn / kKStages) & 1;
-    if (!(ok = wait_bar_warp(&S->v_full[vs], vph, S, p.status))) break;
-    if (!(ok = wait_bar_warp(&S->p_full[0], j & 1, S, p.status))) break;
-    tc_fence_after();
-    pv(0, vs, j > 0);
-    if (jn < n) {
-      if (!(ok = wait_bar_warp(&S->k_full[stn], phn, S, p.status))) break;
-      tc_fence_after();
-      qk(0, stn);
+  ok = ok && wait_bar_warp(&S->q_full, 0, S, p.status);
+  // Issue order per key tile j: QK_0(j), PV_0(j-1), QK_1(j), PV_1(j-1).  A
+  // tile's PV runs one key tile behind its QK^T, so the softmax of S_t(j)
+  // has the MMAs of three other steps (about 2000 clk) to produce P_t(j)
+  // before the pipe needs it, while S, which only has to survive until the
+  // softmax has loaded it, alternates between the tiles.
+  for (int j = 0; ok && j <= n; ++j) {
+    const bool has_qk = j < n;
+    const int st = j % kKStages;
+    const uint32_t ph = (j / kKStages) & 1;
+    const int jp = j - 1;  // the key tile whose PV runs now
+    const int vs = jp % kVStages;
+    const uint32_t vph = (jp / kVStages) & 1;
+    if (has_qk) {
+      if (!(ok = wait_bar_warp(&S->k_full[st], ph, S, p.status) && take_s()))
+        break;
+      qk(0, st);
       mma_commit_warp(&S->s_full[0]);
+      if (!two) mma_commit_warp(&S->k_empty[st]);
+    }
+    if (jp >= 0) {
+      if (!(ok = wait_bar_warp(&S->v_full[vs], vph, S, p.status) &&
+                 wait_bar_warp(&S->p_full[0], jp & 1, S, p.status)))
+        break;
+      tc_fence_after();
+      pv(0, vs, jp > 0);
+      mma_commit_warp(&S->p_free[0]);
+      if (!two) mma_commit_warp(&S->v_empty[vs]);
     }
     if (two) {
-      if (!(ok = wait_bar_warp(&S->p_full[1], j & 1, S, p.status))) break;
-      tc_fence_after();
-      pv(1, vs, j > 0);
-    }
-    mma_commit_warp(&S->v_empty[vs]);
-    if (jn < n) {
-      if (two) {
-        qk(1, stn);
+      if (has_qk) {
+        if (!(ok = take_s())) break;
+        qk(1, st);
         mma_commit_warp(&S->s_full[1]);
+        mma_commit_warp(&S->k_empty[st]);
       }
-      mma_commit_warp(&S->k_empty[stn]);
+      if (jp >= 0) {
+        if (!(ok = wait_bar_warp(&S->p_full[1], jp & 1, S, p.status))) break;
+        tc_fence_after();
+        pv(1, vs, jp > 0);
+        mma_commit_warp(&S->p_free[1]);
+        mma_commit_warp(&S->v_empty[vs]);
+      }
     }
   }
   if (ok) mma_commit_warp(&S->o_full);
@@ -421,12 +442,12 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 }
 
 // P = 2^(s * scale_log2 - m) for the 32 columns of s[c] (a packed FFMA per
-// pair, one MUFU ex2 per element), stored as 16 bf16 pairs at TMEM column
-// tS + 16 c; the row sums go to four independent packed accumulators.
-__device__ __forceinline__ void exp_store32(const uint32_t (&sc)[32],
-                                            uint64_t sl2x2, uint64_t neg2,
-                                            uint32_t taddr, uint64_t (&acc)[4]) {
-  uint32_t pk[16];
+// pair, one MUFU ex2 per element), packed as 16 bf16 pairs; the row sums go
+// to four independent packed accumulators.
+__device__ __forceinline__ void exp_pack32(const uint32_t (&sc)[32],
+                                           uint64_t sl2x2, uint64_t neg2,
+                                           uint32_t (&pk)[16],
+                                           uint64_t (&acc)[4]) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     const uint64_t x2 = f2_fma(f2_pack(__uint_as_float(sc[2 * i]),
@@ -438,7 +459,6 @@ __device__ __forceinline__ void exp_store32(const uint32_t (&sc)[32],
     acc[i & 3] = f2_add(acc[i & 3], f2_pack(p0, p1));
     pk[i] = pack_bf16(p0, p1);
   }
-  tmem_st16(taddr, pk);
 }
 
 __device__ __forceinline__ float acc_total(const uint64_t (&acc)[4]) {
@@ -484,13 +504,18 @@ __device__ __forceinline__ void mask_range_max32(uint32_t (&sc)[32], int c,
 // Streaming: j0, n index the launch's visible tiles.  One-shot: the tiles of
 // [kv0, kv1); a row of chunk c sees keys of chunks max(0, c - W) .. c, so a
 // row can be fully masked in a tile (its reference then stays at -inf).
+// Per key tile: read S (shared by both query tiles) into registers and
+// release it at once, exponentiate, wait until the previous PV of this tile
+// has consumed P_t (and brought O_t up to date), rescale O_t if the
+// reference moved, then store P_t.
 template <int D, bool kOneShot>
 __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
                              int t, int wq, int lane, int j0, int n, int kv0,
                              int kv1, int q0) {
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-  const uint32_t tS = tmem + t * 128 + lane_off;
-  const uint32_t tO = tmem + 256 + t * 128 + lane_off;
+  const uint32_t tS = tmem + kTmemS + lane_off;
+  const uint32_t tP = tmem + kTmemP + t * 64 + lane_off;
+  const uint32_t tO = tmem + kTmemO + t * 128 + lane_off;
   const float sl2 = p.scale_log2;
   const uint64_t sl2x2 = f2_pack(sl2, sl2);
   float m_ref = -INFINITY;  // exp2-domain reference (scaled scores)
@@ -512,26 +537,22 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     if (!(ok = wait_bar(&S->s_full[t], j & 1, S, p.status))) break;
     tc_fence_after();
     uint32_t s[4][32];
-    tmem_ld32(tS + 0, s[0]);
-    tmem_ld32(tS + 32, s[1]);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32 * c, s[c]);
     tmem_wait_ld();
-    tmem_ld32(tS + 64, s[2]);  // lands while the first half is reduced
-    tmem_ld32(tS + 96, s[3]);
+    // S is in registers: the next QK^T (of either tile) may overwrite it.
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&S->s_free);
     float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
     if (kOneShot) {
       const int lo = vis_lo - tok0;
       const int hi = min(vis_hi - tok0, valid);
-      mask_range_max32(s[0], 0, lo, hi, mx);
-      mask_range_max32(s[1], 1, lo, hi, mx);
-      tmem_wait_ld();
-      mask_range_max32(s[2], 2, lo, hi, mx);
-      mask_range_max32(s[3], 3, lo, hi, mx);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) mask_range_max32(s[c], c, lo, hi, mx);
     } else {
-      mask_max32(s[0], 0, valid, mx);
-      mask_max32(s[1], 1, valid, mx);
-      tmem_wait_ld();
-      mask_max32(s[2], 2, valid, mx);
-      mask_max32(s[3], 3, valid, mx);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) mask_max32(s[c], c, valid, mx);
     }
     const float mrow = fmaxf(max3(mx[0], mx[1], mx[2]), mx[3]) * sl2;
     // The reference moves only when a row max passes it by more than the
@@ -550,22 +571,36 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     const float neg = (kOneShot && m_ref == -INFINITY) ? 0.f : -m_ref;
     const uint64_t neg2 = f2_pack(neg, neg);
     uint64_t acc[4] = {0, 0, 0, 0};
+    uint32_t pk[2][16];
 #pragma unroll
-    for (int c = 0; c < 4; ++c) exp_store32(s[c], sl2x2, neg2, tS + 16 * c, acc);
-    l += acc_total(acc);
+    for (int c = 0; c < 2; ++c) exp_pack32(s[c], sl2x2, neg2, pk[c], acc);
+    // P_t(j - 1) has been consumed and O_t holds PV_t(0 .. j-1) (PV_t(j-1)
+    // was issued right after this S, so this normally does not wait).
+    if (j > 0 && !(ok = wait_bar(&S->p_free[t], (j - 1) & 1, S, p.status)))
+      break;
+    tc_fence_after();
     if (rescale && j > 0) {
-      // O_t holds PV_t(0..j-1) and PV_t(j) waits for p_full: scale in place.
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tO + c * 32, r);
+      // Scale O_t in place before PV_t(j) accumulates against the new
+      // reference.
+#pragma unroll 1
+      for (int c = 0; c < D / 8; ++c) {
+        uint32_t r[8];
+        tmem_ld8(tO + c * 8, r);
         tmem_wait_ld();
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
+        for (int i = 0; i < 8; ++i)
           r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-        tmem_st32(tO + c * 32, r);
+        tmem_st8(tO + c * 8, r);
       }
     }
+    tmem_st16(tP, pk[0]);
+    tmem_st16(tP + 16, pk[1]);
+#pragma unroll
+    for (int c = 2; c < 4; ++c) {
+      exp_pack32(s[c], sl2x2, neg2, pk[c - 2], acc);
+      tmem_st16(tP + 16 * c, pk[c - 2]);
+    }
+    l += acc_total(acc);
     tmem_wait_st();
     tc_fence_before();
     // One arrival per warp (lane 0, after the warp's stores are complete):
@@ -726,7 +761,9 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     for (int t = 0; t < kQTiles; ++t) {
       mbar_init(&S->s_full[t], 1);
       mbar_init(&S->p_full[t], 4);
+      mbar_init(&S->p_free[t], 1);
     }
+    mbar_init(&S->s_free, 4);
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
