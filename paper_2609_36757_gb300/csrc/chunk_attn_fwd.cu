@@ -668,21 +668,28 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
 
 // Merge the partial results of the split units: weights 2^(lse_i - m),
 // O = sum_i w_i O_i / sum_i w_i, LSE = m + log2(sum_i w_i) (natural log out).
-// A CTA merges 32 query rows of one unit: thread (r, g) accumulates columns
-// [16 g, 16 g + 16) of row r, so a warp reads 32 consecutive rows of one
-// column of a part (coalesced); the bf16 rows are then written contiguously
-// through shared memory.
+// A CTA merges a block of 32 query rows x 32 columns of one unit: thread
+// (r, g) accumulates columns [4 g, 4 g + 4) of the block for row r, so a
+// warp reads 32 consecutive rows of one column of a part (coalesced).  The
+// parts are walked kPartUnroll at a time with all their loads issued
+// together: the merge reads tens of MB that are mostly still in L2, and it
+// is the latency of those reads, not their volume, that sets its time.  The
+// bf16 rows are written contiguously through shared memory.
 constexpr int kMergeRows = 32;
+constexpr int kMergeCols = 32;
+constexpr int kMergeThreads = kMergeRows * kMergeCols / 4;  // 256
+constexpr int kPartUnroll = 8;
 
 template <int D>
-__global__ void __launch_bounds__(kMergeRows * D / 16)
+__global__ void __launch_bounds__(kMergeThreads)
 combine_kernel(const __grid_constant__ TcParams p) {
-  constexpr int kCols = 16;  // columns per thread
-  __shared__ __align__(16) uint16_t tile[kMergeRows][D + 8];
+  constexpr int kCols = 4;  // columns per thread
+  __shared__ __align__(16) uint16_t tile[kMergeRows][kMergeCols + 8];
   const int ut = blockIdx.x;
   const int r = threadIdx.x % kMergeRows;
   const int g = threadIdx.x / kMergeRows;
   const int r_unit = blockIdx.y * kMergeRows + r;
+  const int col0 = blockIdx.z * kMergeCols + g * kCols;
   const int unit = p.units_full + ut;
   const int pair = unit % p.q_pairs;
   const int h = (unit / p.q_pairs) % p.heads;
@@ -692,23 +699,39 @@ combine_kernel(const __grid_constant__ TcParams p) {
   const int k0 = ut * p.split;
   // every part this block reads lies in the workspace
   if (!in_bounds(k0 + p.split - 1, p.ws_parts, p.status)) return;
+  const float* lse = p.ws_lse + (size_t)k0 * kUnitRows + r_unit;
   float m = -INFINITY;
-  for (int i = 0; i < p.split; ++i)
-    m = fmaxf(m, p.ws_lse[(size_t)(k0 + i) * kUnitRows + r_unit]);
+  for (int i0 = 0; i0 < p.split; i0 += kPartUnroll) {
+    float l8[kPartUnroll];
+#pragma unroll
+    for (int u = 0; u < kPartUnroll; ++u)
+      l8[u] = i0 + u < p.split ? lse[(size_t)(i0 + u) * kUnitRows] : -INFINITY;
+#pragma unroll
+    for (int u = 0; u < kPartUnroll; ++u) m = fmaxf(m, l8[u]);
+  }
   float acc[kCols];
 #pragma unroll
   for (int x = 0; x < kCols; ++x) acc[x] = 0.f;
   float wsum = 0.f;
-  for (int i = 0; i < p.split; ++i) {
-    const float wi = ex2(p.ws_lse[(size_t)(k0 + i) * kUnitRows + r_unit] - m);
-    wsum += wi;
-    const float* src =
-        p.ws + ((size_t)(k0 + i) * D + g * kCols) * kUnitRows + r_unit;
-    float v[kCols];
+  const float* src0 = p.ws + ((size_t)k0 * D + col0) * kUnitRows + r_unit;
+  for (int i0 = 0; i0 < p.split; i0 += kPartUnroll) {
+    float w8[kPartUnroll], v[kPartUnroll][kCols];
 #pragma unroll
-    for (int x = 0; x < kCols; ++x) v[x] = src[x * kUnitRows];
+    for (int u = 0; u < kPartUnroll; ++u) {
+      const bool have = i0 + u < p.split;
+      w8[u] = have ? lse[(size_t)(i0 + u) * kUnitRows] : -INFINITY;
+      const float* src = src0 + (size_t)(i0 + u) * D * kUnitRows;
 #pragma unroll
-    for (int x = 0; x < kCols; ++x) acc[x] = fmaf(wi, v[x], acc[x]);
+      for (int x = 0; x < kCols; ++x)
+        v[u][x] = have ? src[(size_t)x * kUnitRows] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < kPartUnroll; ++u) {
+      const float wi = ex2(w8[u] - m);  // 0 for the missing parts
+      wsum += wi;
+#pragma unroll
+      for (int x = 0; x < kCols; ++x) acc[x] = fmaf(wi, v[u][x], acc[x]);
+    }
   }
   const float inv = 1.f / wsum;
 #pragma unroll
@@ -716,16 +739,19 @@ combine_kernel(const __grid_constant__ TcParams p) {
     *reinterpret_cast<uint32_t*>(&tile[r][g * kCols + x]) =
         pack_bf16(acc[x] * inv, acc[x + 1] * inv);
   const int64_t lse_i = ((int64_t)b * p.heads + h) * p.q_tokens + row0 + r;
-  if (g == 0 && p.lse != nullptr && row0 + r < p.q_tokens &&
+  if (blockIdx.z == 0 && g == 0 && p.lse != nullptr && row0 + r < p.q_tokens &&
       in_bounds(lse_i, (int64_t)p.batch * p.heads * p.q_tokens, p.status))
     p.lse[lse_i] = (m + __log2f(wsum)) * 0.6931471805599453f;
   __syncthreads();
-  // Each row is d bf16 = D / 8 16-byte pieces; one piece per thread.
-  for (int i = threadIdx.x; i < kMergeRows * D / 8; i += blockDim.x) {
-    const int rr = i / (D / 8), piece = i % (D / 8);
+  // Each row of the block is 32 bf16 = 4 16-byte pieces; one piece per
+  // thread of the first 128.
+  if (threadIdx.x < kMergeRows * kMergeCols / 8) {
+    const int rr = threadIdx.x / (kMergeCols / 8);
+    const int piece = threadIdx.x % (kMergeCols / 8);
     const int row = row0 + rr;
     const int64_t x = (int64_t)b * p.o_str.batch + (int64_t)row * p.o_str.token +
-                      (int64_t)h * p.o_str.head + piece * 8;
+                      (int64_t)h * p.o_str.head + blockIdx.z * kMergeCols +
+                      piece * 8;
     if (row < p.q_tokens && in_bounds(x, p.o_elems - 7, p.status))
       *reinterpret_cast<uint4*>(p.o + x) =
           *reinterpret_cast<const uint4*>(&tile[rr][piece * 8]);
@@ -905,8 +931,9 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
   chunk_attn_tc_kernel<D, false><<<grid, kThreads, smem, stream>>>(p);
   *launches = 1;
   if (p.split > 1) {
-    combine_kernel<D><<<dim3(units - p.units_full, kUnitRows / kMergeRows),
-                        kMergeRows * D / 16, 0, stream>>>(p);
+    combine_kernel<D><<<dim3(units - p.units_full, kUnitRows / kMergeRows,
+                             D / kMergeCols),
+                        kMergeThreads, 0, stream>>>(p);
     *launches = 2;
   }
   return cudaGetLastError();

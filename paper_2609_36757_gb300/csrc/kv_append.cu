@@ -45,20 +45,22 @@ __global__ void __launch_bounds__(256) kv_append_kernel(AppendParams p) {
   const uint32_t n = (uint32_t)p.batch * p.tokens * p.heads * VPR;
   const int64_t cache_vecs = (int64_t)p.batch * p.heads * p.cache_tokens * VPR;
   const uint32_t stride = gridDim.x * blockDim.x;
-  uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
-  for (; i + (kUnroll - 1) * stride < n; i += kUnroll * stride) {
+  // Every pass issues all of its (predicated) loads before the first store,
+  // also the last, partial one: a small chunk gives each thread only a few
+  // vectors, and one load at a time would leave it latency-bound.  Indices
+  // stay below n + kUnroll * stride, which the launch keeps within 32 bits.
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += kUnroll * stride) {
     uint4 v[kUnroll];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) v[u] = __ldcs(src + i + u * stride);
+    for (int u = 0; u < kUnroll; ++u)
+      if (i + u * stride < n) v[u] = __ldcs(src + i + u * stride);
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
+      if (i + u * stride >= n) break;
       const int64_t c = cache_index<VPR>(p, i + u * stride);
       if (in_bounds(c, cache_vecs, p.status)) dst[c] = v[u];
     }
-  }
-  for (; i < n; i += stride) {
-    const int64_t c = cache_index<VPR>(p, i);
-    if (in_bounds(c, cache_vecs, p.status)) dst[c] = __ldcs(src + i);
   }
 }
 
@@ -69,6 +71,7 @@ cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream) {
   const int64_t n = (int64_t)p.batch * p.tokens * p.heads * vpr;
   if (n == 0) return cudaSuccess;
   if (n > 0x7fffffffLL) return cudaErrorInvalidValue;  // 32-bit indexing
+  // (n < 2^31 and kUnroll * stride < 2^31: i + u * stride never wraps)
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
