@@ -685,6 +685,8 @@ __global__ void __launch_bounds__(kMergeThreads)
 combine_kernel(const __grid_constant__ TcParams p) {
   constexpr int kCols = 4;  // columns per thread
   __shared__ __align__(16) uint16_t tile[kMergeRows][kMergeCols + 8];
+  pdl_trigger();
+  pdl_wait();  // the partial results of the attention kernel are complete
   const int ut = blockIdx.x;
   const int r = threadIdx.x % kMergeRows;
   const int g = threadIdx.x / kMergeRows;
@@ -800,6 +802,10 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = S->tmem_base;
+  // Set-up above touched no global memory; Q, K, V and the outputs may
+  // belong to the previous kernel on the stream until it has completed.
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 8) {
     if (lane == 0) producer<D, true, kOneShot>(p, smem, S, w);
@@ -928,15 +934,19 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
       chunk_attn_tc_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
       smem);
   if (e != cudaSuccess) return e;
-  chunk_attn_tc_kernel<D, false><<<grid, kThreads, smem, stream>>>(p);
+  e = launch_pdl(chunk_attn_tc_kernel<D, false>, dim3(grid), dim3(kThreads),
+                 smem, stream, p);
+  if (e != cudaSuccess) return e;
   *launches = 1;
   if (p.split > 1) {
-    combine_kernel<D><<<dim3(units - p.units_full, kUnitRows / kMergeRows,
-                             D / kMergeCols),
-                        kMergeThreads, 0, stream>>>(p);
+    e = launch_pdl(combine_kernel<D>,
+                   dim3(units - p.units_full, kUnitRows / kMergeRows,
+                        D / kMergeCols),
+                   dim3(kMergeThreads), 0, stream, p);
+    if (e != cudaSuccess) return e;
     *launches = 2;
   }
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // One unit per pair of query tiles, no key splitting: the units differ in
@@ -981,8 +991,8 @@ cudaError_t launch_oneshot_d(const OneShotParams& a, cudaStream_t stream) {
       chunk_attn_tc_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
       smem);
   if (e != cudaSuccess) return e;
-  chunk_attn_tc_kernel<D, true><<<grid, kThreads, smem, stream>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(chunk_attn_tc_kernel<D, true>, dim3(grid), dim3(kThreads),
+                    smem, stream, p);
 }
 
 }  // namespace

@@ -59,6 +59,40 @@ __device__ __forceinline__ bool in_bounds(int64_t, int64_t, int*) {
 #endif
 #endif
 
+#ifdef __CUDACC__
+// Programmatic dependent launch.  The streaming kernels (append, attention,
+// split merge) and the one-step update are launched with programmatic stream
+// serialization, so a kernel may become resident and do its set-up (barrier
+// and TMEM initialisation) while the previous kernel on the stream drains.
+// Each of them executes pdl_wait() before its first global-memory access
+// that a preceding kernel may produce or still read (the wait returns once
+// that kernel has completed and its writes are visible), and pdl_trigger()
+// early, so that the next kernel's launch can begin.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                              size_t smem, cudaStream_t stream,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+#endif
+
 // Strided view of a bfloat16 [B, L, H, d] token-major tensor or of a head-major
 // cache [B, H, L, d]: element (b, t, h, x) lives at
 // base + b*batch + t*token + h*head + x (strides in elements).

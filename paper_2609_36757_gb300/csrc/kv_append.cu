@@ -39,6 +39,8 @@ __device__ __forceinline__ int64_t cache_index(const AppendParams& p,
 // blockIdx.y selects K (0) or V (1).
 template <int VPR>
 __global__ void __launch_bounds__(256) kv_append_kernel(AppendParams p) {
+  pdl_trigger();
+  pdl_wait();  // the chunk's K/V and the slot's previous readers are done
   const uint4* src =
       reinterpret_cast<const uint4*>(blockIdx.y ? p.v_new : p.k_new);
   uint4* dst = reinterpret_cast<uint4*>(blockIdx.y ? p.v_cache : p.k_cache);
@@ -82,12 +84,10 @@ cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t stream) {
   if (blocks > need) blocks = need;
   const dim3 grid((unsigned)blocks, 2);
   if (vpr == 16)
-    kv_append_kernel<16><<<grid, 256, 0, stream>>>(p);
-  else if (vpr == 8)
-    kv_append_kernel<8><<<grid, 256, 0, stream>>>(p);
-  else
-    return cudaErrorInvalidValue;
-  return cudaGetLastError();
+    return launch_pdl(kv_append_kernel<16>, grid, dim3(256), 0, stream, p);
+  if (vpr == 8)
+    return launch_pdl(kv_append_kernel<8>, grid, dim3(256), 0, stream, p);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace fastvr

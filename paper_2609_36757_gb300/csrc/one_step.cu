@@ -59,6 +59,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
 one_step_kernel(const T* z, const __nv_bfloat16* __restrict__ v, T* out,
                 int64_t n, float neg_sigma) {
+  pdl_trigger();
+  pdl_wait();  // z and v may come from the previous kernel on the stream
   const int64_t n8 = n / 8;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -99,16 +101,17 @@ cudaError_t launch_one_step(const void* z, const void* v, void* out, int64_t n,
   int64_t blocks = (int64_t)sms * 8;
   const int64_t need = (n / 8 + 255) / 256 + 1;
   if (blocks > need) blocks = need;
+  const float neg_sigma = -sigma;
   if (dtype == 0)
-    one_step_kernel<__nv_bfloat16><<<(unsigned)blocks, 256, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(z),
-        static_cast<const __nv_bfloat16*>(v), static_cast<__nv_bfloat16*>(out),
-        n, -sigma);
-  else
-    one_step_kernel<float><<<(unsigned)blocks, 256, 0, stream>>>(
-        static_cast<const float*>(z), static_cast<const __nv_bfloat16*>(v),
-        static_cast<float*>(out), n, -sigma);
-  return cudaGetLastError();
+    return launch_pdl(one_step_kernel<__nv_bfloat16>, dim3((unsigned)blocks),
+                      dim3(256), 0, stream,
+                      static_cast<const __nv_bfloat16*>(z),
+                      static_cast<const __nv_bfloat16*>(v),
+                      static_cast<__nv_bfloat16*>(out), n, neg_sigma);
+  return launch_pdl(one_step_kernel<float>, dim3((unsigned)blocks), dim3(256),
+                    0, stream, static_cast<const float*>(z),
+                    static_cast<const __nv_bfloat16*>(v),
+                    static_cast<float*>(out), n, neg_sigma);
 }
 
 }  // namespace fastvr
