@@ -63,6 +63,12 @@ constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleThreshold = 8.0f;      // log2 units
 constexpr int kMinTilesPerPart = 4;             // key tiles per split part
 constexpr uint64_t kDefaultWaitLimitNs = 4000000000ull;  // 4 s per wait
+// Named (hardware) barriers of the softmax -> MMA hand-offs: S read (free
+// for the next QK^T) and P_t stored.  The four softmax warps of a tile
+// arrive, the MMA warp syncs: kHandoff threads per generation.
+constexpr int kBarSFree = 1;
+constexpr int kBarPFull0 = 2;  // + t
+constexpr int kHandoff = 5 * 32;
 
 struct TcParams {
   CUtensorMap q_map;                  // {d, Lq, H, B}
@@ -165,8 +171,7 @@ struct Shared {
   uint64_t q_full;
   uint64_t k_full[kKStages], k_empty[kKStages];
   uint64_t v_full[kVStages], v_empty[kVStages];
-  uint64_t s_full[kQTiles], p_full[kQTiles], p_free[kQTiles];
-  uint64_t s_free;
+  uint64_t s_full[kQTiles], p_free[kQTiles];
   uint64_t o_full, drain;
   uint32_t tmem_base;
   int abort;
@@ -309,6 +314,20 @@ __device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity,
   }
 }
 
+// Hand-offs from the softmax warps to the MMA warp go through named
+// barriers, which live in hardware rather than in shared memory: an mbarrier
+// poll is a shared-memory access, and while SMEM x SMEM MMAs are queued every
+// such access waits behind their operand reads (~200 clk), which the issuer
+// cannot afford several times per key tile.  A named barrier has no time
+// limit, so the softmax warps make exactly the arrivals the MMA warp will
+// wait for on every path, also after a failed wait (see softmax_role).
+__device__ __forceinline__ void named_arrive(int id) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "n"(kHandoff) : "memory");
+}
+__device__ __forceinline__ void named_sync(int id) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kHandoff) : "memory");
+}
+
 template <int D>
 __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
                            uint32_t tmem, const Work& w) {
@@ -352,12 +371,11 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
                   (acc | kk) != 0);
   };
   // The k-th QK^T (of either tile) may overwrite S once the softmax warps
-  // have read the previous one into registers (completion k - 1 of s_free).
+  // have read the previous one into registers (generation k - 1 of the S
+  // barrier).
   int s_uses = 0;
   auto take_s = [&]() -> bool {
-    if (s_uses > 0 &&
-        !wait_bar_warp(&S->s_free, (uint32_t)(s_uses - 1) & 1, S, p.status))
-      return false;
+    if (s_uses > 0) named_sync(kBarSFree);
     ++s_uses;
     tc_fence_after();
     return true;
@@ -387,9 +405,8 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
       if (!two) mma_commit_warp(&S->k_empty[st]);
     }
     if (jp >= 0) {
-      if (!(ok = wait_bar_warp(&S->v_full[vs], vph, S, p.status) &&
-                 wait_bar_warp(&S->p_full[0], jp & 1, S, p.status)))
-        break;
+      if (!(ok = wait_bar_warp(&S->v_full[vs], vph, S, p.status))) break;
+      named_sync(kBarPFull0);
       tc_fence_after();
       pv(0, vs, jp > 0);
       mma_commit_warp(&S->p_free[0]);
@@ -403,7 +420,7 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
         mma_commit_warp(&S->k_empty[st]);
       }
       if (jp >= 0) {
-        if (!(ok = wait_bar_warp(&S->p_full[1], jp & 1, S, p.status))) break;
+        named_sync(kBarPFull0 + 1);
         tc_fence_after();
         pv(1, vs, jp > 0);
         mma_commit_warp(&S->p_free[1]);
@@ -510,8 +527,8 @@ __device__ __forceinline__ void mask_range_max32(uint32_t (&sc)[32], int c,
 // reference moved, then store P_t.
 template <int D, bool kOneShot>
 __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
-                             int t, int wq, int lane, int j0, int n, int kv0,
-                             int kv1, int q0) {
+                             int t, int nqt, int wq, int lane, int j0, int n,
+                             int kv0, int kv1, int q0) {
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
   const uint32_t tS = tmem + kTmemS + lane_off;
   const uint32_t tP = tmem + kTmemP + t * 64 + lane_off;
@@ -521,6 +538,10 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   float m_ref = -INFINITY;  // exp2-domain reference (scaled scores)
   float l = 0.f;
   bool ok = true;
+  // Arrivals the MMA warp waits for: one per S this tile reads, except the
+  // very last S of the unit (no QK^T follows it), and one per P_t.
+  const int s_expected = (t == nqt - 1) ? n - 1 : n;
+  int s_arrived = 0, p_arrived = 0;
   int vis_lo = 0, vis_hi = 0;  // one-shot: this row's visible key tokens
   if (kOneShot) {
     const int row = min(q0 + t * kBM + wq * 32 + lane, p.q_tokens - 1);
@@ -542,8 +563,10 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     tmem_wait_ld();
     // S is in registers: the next QK^T (of either tile) may overwrite it.
     tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&S->s_free);
+    if (s_arrived < s_expected) {
+      named_arrive(kBarSFree);
+      ++s_arrived;
+    }
     float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
     if (kOneShot) {
       const int lo = vis_lo - tok0;
@@ -603,11 +626,19 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     l += acc_total(acc);
     tmem_wait_st();
     tc_fence_before();
-    // One arrival per warp (lane 0, after the warp's stores are complete):
-    // the barrier word sits in shared memory, which queued QK^T MMAs keep
-    // busy, so 32 arrivals per warp would each wait their turn.
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&S->p_full[t]);
+    named_arrive(kBarPFull0 + t);
+    ++p_arrived;
+  }
+  // After a failed wait the remaining hand-offs are still made (their
+  // contents are undefined, and so is the output), so that the MMA warp
+  // never waits for an arrival that does not come.
+  while (s_arrived < s_expected) {
+    named_arrive(kBarSFree);
+    ++s_arrived;
+  }
+  while (p_arrived < n) {
+    named_arrive(kBarPFull0 + t);
+    ++p_arrived;
   }
   if (!ok || !wait_bar(&S->o_full, 0, S, p.status)) return;
   tc_fence_after();
@@ -788,10 +819,8 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     }
     for (int t = 0; t < kQTiles; ++t) {
       mbar_init(&S->s_full[t], 1);
-      mbar_init(&S->p_full[t], 4);
       mbar_init(&S->p_free[t], 1);
     }
-    mbar_init(&S->s_free, 4);
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -818,8 +847,8 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
   } else {
     // A query tile that lies past the end of the chunk has no work.
     if (warp / 4 < w.nqt)
-      softmax_role<D, kOneShot>(p, S, tmem, warp / 4, warp % 4, lane, w.j0,
-                                w.n, w.kv0, w.kv1, w.q0);
+      softmax_role<D, kOneShot>(p, S, tmem, warp / 4, w.nqt, warp % 4, lane,
+                                w.j0, w.n, w.kv0, w.kv1, w.q0);
   }
   tc_fence_before();
   __syncthreads();
