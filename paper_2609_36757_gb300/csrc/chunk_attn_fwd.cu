@@ -52,7 +52,8 @@ constexpr int kBN = 128;        // keys per tile
 constexpr int kQTiles = 2;      // query tiles per CTA
 constexpr int kKStages = 3;     // depth of the K ring
 constexpr int kVStages = 2;     // depth of the V ring
-constexpr int kThreads = 352;   // 8 softmax warps, K and V producers, MMA
+constexpr int kThreads = 384;   // 8 softmax warps, K and V producers, MMA,
+                                // relay
 constexpr int kBox = 128 * 128; // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns: one S tile shared by the two query tiles, P_0 and P_1 (bf16
@@ -69,6 +70,11 @@ constexpr uint64_t kDefaultWaitLimitNs = 4000000000ull;  // 4 s per wait
 constexpr int kBarSFree = 1;
 constexpr int kBarPFull0 = 2;  // + t
 constexpr int kHandoff = 5 * 32;
+// Named barriers of the relay -> MMA hand-offs, one per ring stage: K (or V)
+// stage s has landed.  The relay warp arrives, the MMA warp syncs.
+constexpr int kBarKFull0 = 4;  // + stage (kKStages of them)
+constexpr int kBarVFull0 = 7;  // + stage (kVStages of them)
+constexpr int kRelay = 2 * 32;
 
 struct TcParams {
   CUtensorMap q_map;                  // {d, Lq, H, B}
@@ -327,6 +333,45 @@ __device__ __forceinline__ void named_arrive(int id) {
 __device__ __forceinline__ void named_sync(int id) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kHandoff) : "memory");
 }
+__device__ __forceinline__ void relay_arrive(int id) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "n"(kRelay) : "memory");
+}
+__device__ __forceinline__ void relay_sync(int id) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kRelay) : "memory");
+}
+
+// The relay warp observes the TMA completions in the order the MMA warp
+// needs them (K(j), then V(j - 1)) and hands each over through the named
+// barrier of its ring stage, so the MMA warp itself never polls a
+// shared-memory barrier.  A stage's barrier cannot be arrived at twice
+// before the MMA warp has synced on it: the producer refills the stage only
+// after the MMAs that read it.  After a failed wait the remaining arrivals
+// are still made (the MMA warp then computes on undefined data, and the
+// failure is recorded), so the MMA warp never waits for one that does not
+// come.
+__device__ void relay_role(const TcParams& p, Shared* S, int n) {
+  int k_arr = 0, v_arr = 0;
+  bool ok = true;
+  for (int j = 0; ok && j <= n; ++j) {
+    if (j < n) {
+      if (!(ok = wait_bar_warp(&S->k_full[j % kKStages], (j / kKStages) & 1,
+                               S, p.status)))
+        break;
+      relay_arrive(kBarKFull0 + j % kKStages);
+      ++k_arr;
+    }
+    const int jp = j - 1;
+    if (jp >= 0) {
+      if (!(ok = wait_bar_warp(&S->v_full[jp % kVStages],
+                               (jp / kVStages) & 1, S, p.status)))
+        break;
+      relay_arrive(kBarVFull0 + jp % kVStages);
+      ++v_arr;
+    }
+  }
+  for (; k_arr < n; ++k_arr) relay_arrive(kBarKFull0 + k_arr % kKStages);
+  for (; v_arr < n; ++v_arr) relay_arrive(kBarVFull0 + v_arr % kVStages);
+}
 
 template <int D>
 __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
@@ -374,11 +419,10 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   // have read the previous one into registers (generation k - 1 of the S
   // barrier).
   int s_uses = 0;
-  auto take_s = [&]() -> bool {
+  auto take_s = [&]() {
     if (s_uses > 0) named_sync(kBarSFree);
     ++s_uses;
     tc_fence_after();
-    return true;
   };
 
   // Test hook: o_full receives no arrival before the end of the stream, so
@@ -393,19 +437,17 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
   for (int j = 0; ok && j <= n; ++j) {
     const bool has_qk = j < n;
     const int st = j % kKStages;
-    const uint32_t ph = (j / kKStages) & 1;
     const int jp = j - 1;  // the key tile whose PV runs now
     const int vs = jp % kVStages;
-    const uint32_t vph = (jp / kVStages) & 1;
     if (has_qk) {
-      if (!(ok = wait_bar_warp(&S->k_full[st], ph, S, p.status) && take_s()))
-        break;
+      relay_sync(kBarKFull0 + st);
+      take_s();
       qk(0, st);
       mma_commit_warp(&S->s_full[0]);
       if (!two) mma_commit_warp(&S->k_empty[st]);
     }
     if (jp >= 0) {
-      if (!(ok = wait_bar_warp(&S->v_full[vs], vph, S, p.status))) break;
+      relay_sync(kBarVFull0 + vs);
       named_sync(kBarPFull0);
       tc_fence_after();
       pv(0, vs, jp > 0);
@@ -414,7 +456,7 @@ __device__ void mma_issuer(const TcParams& p, uint8_t* smem, Shared* S,
     }
     if (two) {
       if (has_qk) {
-        if (!(ok = take_s())) break;
+        take_s();
         qk(1, st);
         mma_commit_warp(&S->s_full[1]);
         mma_commit_warp(&S->k_empty[st]);
@@ -844,6 +886,8 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     __syncwarp();
   } else if (warp == 9) {
     mma_issuer<D>(p, smem, S, tmem, w);
+  } else if (warp == 11) {
+    relay_role(p, S, w.n);
   } else {
     // A query tile that lies past the end of the chunk has no work.
     if (warp / 4 < w.nqt)
