@@ -45,9 +45,23 @@ constexpr int kStages1 = 2;       // ring 1 depth (ring 0: per kernel)
 constexpr int kDkdvS0 = 2;        // dK/dV ring 0 (Q and row vectors)
 constexpr int kDqS0 = 3;          // dQ ring 0 (K): loads one step earlier
 static_assert(kDkdvS0 == kStages1, "dK/dV indexes both rings alike");
-constexpr int kThreads = 320;     // 8 compute warps, producer, MMA issuer
+constexpr int kThreads = 352;     // 8 compute warps, producer, MMA issuer,
+                                  // relay
 constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp = 9;
+constexpr int kRelayWarp = 10;
+// Named (hardware) barriers of the hand-offs to the MMA warp: P stored and
+// dS stored (the eight compute warps arrive, the MMA warp syncs), and one
+// per stage of each streamed ring (the relay warp arrives once the stage's
+// TMA loads have landed, the MMA warp syncs).  An mbarrier poll is a
+// shared-memory access that waits ~200 clk behind queued SMEM x SMEM MMAs;
+// a named barrier whose arrivals are in costs the MMA warp next to nothing.
+constexpr int kBarP = 1;
+constexpr int kBarDS = 2;
+constexpr int kBarRing0 = 3;  // + stage, up to kMaxStages
+constexpr int kBarRing1 = 6;  // + stage, up to kStages1
+constexpr int kComputeHandoff = 9 * 32;
+constexpr int kRelayHandoff = 2 * 32;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
@@ -73,7 +87,7 @@ struct BwdShared {
   // dO, last read by dV), so a ring-1 slot is refilled as soon as its last
   // reader has run instead of waiting for the end of the step.
   uint64_t full[2][kMaxStages], empty[2][kMaxStages];
-  uint64_t s_ready, dp_ready, p_ready, ds_ready, o_full, drain;
+  uint64_t s_ready, dp_ready, o_full, drain;
   uint32_t tmem_base;
   int abort;
   int* status;
@@ -156,6 +170,43 @@ __device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity,
   }
 }
 
+__device__ __forceinline__ void compute_arrive(int id) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "n"(kComputeHandoff) : "memory");
+}
+__device__ __forceinline__ void compute_sync(int id) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kComputeHandoff) : "memory");
+}
+__device__ __forceinline__ void relay_arrive(int id) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "n"(kRelayHandoff) : "memory");
+}
+__device__ __forceinline__ void relay_sync(int id) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kRelayHandoff) : "memory");
+}
+
+// The relay warp observes each step's two streamed tiles (ring 0, then
+// ring 1, the order in which the MMA warp needs them) and hands each stage
+// over through its named barrier.  A stage's barrier cannot be arrived at
+// twice before the MMA warp has synced on it: the producer refills a stage
+// only after the MMAs that read it.  Named barriers have no time limit, so
+// after a failed wait the relay still makes the remaining arrivals (the
+// MMA warp then computes on undefined data; the failure is recorded).
+template <int kS0>
+__device__ void bwd_relay(BwdShared* S, int n) {
+  int a0 = 0, a1 = 0;
+  bool ok = true;
+  for (int j = 0; ok && j < n; ++j) {
+    if (!(ok = wait_bar_warp(&S->full[0][j % kS0], (j / kS0) & 1, S))) break;
+    relay_arrive(kBarRing0 + j % kS0);
+    ++a0;
+    if (!(ok = wait_bar_warp(&S->full[1][j % kStages1], (j / kStages1) & 1, S)))
+      break;
+    relay_arrive(kBarRing1 + j % kStages1);
+    ++a1;
+  }
+  for (; a0 < n; ++a0) relay_arrive(kBarRing0 + a0 % kS0);
+  for (; a1 < n; ++a1) relay_arrive(kBarRing1 + a1 % kStages1);
+}
+
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   const uint64_t t0 = global_timer_ns();
   while (!mbar_try_wait(bar, parity))
@@ -205,12 +256,6 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S,
       }
     mbar_init(&S->s_ready, 1);
     mbar_init(&S->dp_ready, 1);
-    // One arrival per compute warp (lane 0, after the warp's TMEM accesses
-    // are complete): the barrier words sit in shared memory, which queued
-    // SMEM x SMEM MMAs keep saturated, so per-thread arrivals would each
-    // wait their turn.
-    mbar_init(&S->p_ready, 8);
-    mbar_init(&S->ds_ready, 8);
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -452,6 +497,8 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
                             p.lse2 + (int64_t)bh_row(p, b, h) * p.padded,
                             p.delta + (int64_t)bh_row(p, b, h) * p.padded);
     __syncwarp();
+  } else if (warp == kRelayWarp) {
+    bwd_relay<kDkdvS0>(S, n);
   } else if (warp == kMmaWarp) {
     const uint32_t sbase = smem_addr(smem);
     // The next tile's S^T is issued right after this tile's dV (it
@@ -462,35 +509,35 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     // Test hook: o_full receives no arrival before the end, so this wait
     // runs out and exercises the abort path.
     bool ok = (!p.inject_stall || wait_bar_warp(&S->o_full, 0, S)) &&
-              wait_bar_warp(&S->fixed_full, 0, S) &&
-              wait_bar_warp(&S->full[0][0], 0, S) &&
-              wait_bar_warp(&S->full[1][0], 0, S);
+              wait_bar_warp(&S->fixed_full, 0, S);
     if (ok) {
+      relay_sync(kBarRing0);
       tc_fence_after();
       mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S^T_0 = K Q_0^T
       mma_commit_warp(&S->s_ready);
+      relay_sync(kBarRing1);
+      tc_fence_after();
       mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
       mma_commit_warp(&S->dp_ready);
     }
     for (int j = 0; ok && j < n; ++j) {
       const int st = j % kStages1, stn = (j + 1) % kStages1;
-      const uint32_t phn = ((j + 1) / kStages1) & 1;
-      if (!(ok = wait_bar_warp(&S->p_ready, j & 1, S))) break;
+      compute_sync(kBarP);
       tc_fence_after();
       mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
       mma_commit_warp(&S->empty[1][st]);  // dO_j read for the last time
       if (j + 1 < n) {
-        if (!(ok = wait_bar_warp(&S->full[0][stn], phn, S))) break;
+        relay_sync(kBarRing0 + stn);
         tc_fence_after();
         mma_nt<D, L>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
         mma_commit_warp(&S->s_ready);
       }
-      if (!(ok = wait_bar_warp(&S->ds_ready, j & 1, S))) break;
+      compute_sync(kBarDS);
       tc_fence_after();
       mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
       mma_commit_warp(&S->empty[0][st]);  // Q_j and the row vectors
       if (j + 1 < n) {
-        if (!(ok = wait_bar_warp(&S->full[1][stn], phn, S))) break;
+        relay_sync(kBarRing1 + stn);
         tc_fence_after();
         mma_nt<D, L>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
         mma_commit_warp(&S->dp_ready);
@@ -513,6 +560,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     key_sees(p, k0 + t, vis_lo, vis_hi);
     const uint64_t c2x2 = f2(p.scale_log2, p.scale_log2);
     bool ok = true;
+    int p_arr = 0, ds_arr = 0;  // hand-offs made to the MMA warp
     for (int j = 0; j < n; ++j) {
       const int i0 = q0 + j * kT + 64 * hf;  // first query of this half
       const int st = j % kDkdvS0;
@@ -546,8 +594,8 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       tmem_st16(row_t + cs + 16, pb1);
       tmem_wait_st();
       tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&S->p_ready);
+      compute_arrive(kBarP);
+      ++p_arr;
       // phase 2 (overlaps the dV and next S^T MMAs): dS^T over the first
       // half of dP^T; the D values are read ahead like the LSE values
 #pragma unroll
@@ -566,9 +614,14 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&S->ds_ready);
+      compute_arrive(kBarDS);
+      ++ds_arr;
     }
+    // After a failed wait the remaining hand-offs are still made (with
+    // undefined contents), so that the MMA warp never waits for an arrival
+    // that does not come.
+    for (; p_arr < n; ++p_arr) compute_arrive(kBarP);
+    for (; ds_arr < n; ++ds_arr) compute_arrive(kBarDS);
     if (ok && wait_bar_warp(&S->o_full, 0, S)) {
       tc_fence_after();
       const int key = k0 + t;
@@ -616,6 +669,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       bwd_producer<D, false, kDqS0>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map,
                              &p.v_map, kv0, n, h, b, nullptr, nullptr);
     __syncwarp();
+  } else if (warp == kRelayWarp) {
+    bwd_relay<kDqS0>(S, n);
   } else if (warp == kMmaWarp) {
     const uint32_t sbase = smem_addr(smem);
     // S of the next tile is issued as soon as P of this one is in
@@ -623,13 +678,14 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     // Test hook: o_full receives no arrival before the end, so this wait
     // runs out and exercises the abort path.
     bool ok = (!p.inject_stall || wait_bar_warp(&S->o_full, 0, S)) &&
-              wait_bar_warp(&S->fixed_full, 0, S) &&
-              wait_bar_warp(&S->full[0][0], 0, S) &&
-              wait_bar_warp(&S->full[1][0], 0, S);
+              wait_bar_warp(&S->fixed_full, 0, S);
     if (ok) {
+      relay_sync(kBarRing0);
       tc_fence_after();
       mma_nt<D, L>(sbase, tmem, 0, 0, 0, 0);    // S_0 = Q K_0^T
       mma_commit_warp(&S->s_ready);
+      relay_sync(kBarRing1);
+      tc_fence_after();
       mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
       mma_commit_warp(&S->dp_ready);
       mma_commit_warp(&S->empty[1][0]);           // V_0 read for the last time
@@ -638,21 +694,19 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       // K (ring 0) and V (ring 1) run at their own depths
       const int k_st = j % kDqS0, k_stn = (j + 1) % kDqS0;
       const int v_stn = (j + 1) % kStages1;
-      if (!(ok = wait_bar_warp(&S->p_ready, j & 1, S))) break;
+      compute_sync(kBarP);
       if (j + 1 < n) {
-        if (!(ok = wait_bar_warp(&S->full[0][k_stn], ((j + 1) / kDqS0) & 1, S)))
-          break;
+        relay_sync(kBarRing0 + k_stn);
         tc_fence_after();
         mma_nt<D, L>(sbase, tmem, 0, 0, k_stn, 0);  // S_{j+1}
         mma_commit_warp(&S->s_ready);
       }
-      if (!(ok = wait_bar_warp(&S->ds_ready, j & 1, S))) break;
+      compute_sync(kBarDS);
       tc_fence_after();
       mma_tn<D>(sbase, tmem, 256, 128, L::ring(k_st, 0, 0), j > 0);  // dQ
       mma_commit_warp(&S->empty[0][k_st]);  // K_j read for the last time
       if (j + 1 < n) {
-        const uint32_t v_phn = ((j + 1) / kStages1) & 1;
-        if (!(ok = wait_bar_warp(&S->full[1][v_stn], v_phn, S))) break;
+        relay_sync(kBarRing1 + v_stn);
         tc_fence_after();
         mma_nt<D, L>(sbase, tmem, 128, 1, v_stn, 1);  // dP_{j+1}
         mma_commit_warp(&S->dp_ready);
@@ -686,6 +740,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     for (int q = 0; q < 8; ++q) nd_v[q] = make_float4(nd_row, nd_row, nd_row, nd_row);
     const uint64_t c2x2 = f2(p.scale_log2, p.scale_log2);
     bool ok = true;
+    int p_arr = 0, ds_arr = 0;  // hand-offs made to the MMA warp
     for (int j = 0; j < n; ++j) {
       const int tok0 = kv0 + j * kT + 64 * hf;
       if (!(ok = wait_bar_warp(&S->s_ready, j & 1, S))) break;
@@ -703,8 +758,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       p32(x0, nl_v, 0, lo_m, hi_m, need_mask, c2x2, pb0);
       p32(x1, nl_v, 32, lo_m, hi_m, need_mask, c2x2, pb1);
       tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&S->p_ready);
+      compute_arrive(kBarP);
+      ++p_arr;
       // phase 2 (overlaps the next tile's S MMAs): dS over the dP columns
       if (!(ok = wait_bar_warp(&S->dp_ready, j & 1, S))) break;
       tc_fence_after();
@@ -717,9 +772,14 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tmem_st16(row_t + cp + 16, pk);
       tmem_wait_st();
       tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&S->ds_ready);
+      compute_arrive(kBarDS);
+      ++ds_arr;
     }
+    // After a failed wait the remaining hand-offs are still made (with
+    // undefined contents), so that the MMA warp never waits for an arrival
+    // that does not come.
+    for (; p_arr < n; ++p_arr) compute_arrive(kBarP);
+    for (; ds_arr < n; ++ds_arr) compute_arrive(kBarDS);
     if (ok && wait_bar_warp(&S->o_full, 0, S)) {
       tc_fence_after();
       const int64_t off = (int64_t)b * p.seq_tokens * p.heads * D +
