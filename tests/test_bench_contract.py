@@ -47,7 +47,7 @@ def test_reference_arm_line():
 @pytest.mark.gpu
 def test_gpu_arm_line():
     d = _run("--workload", "480p", "--steps", "3", "--warmup", "3",
-             "--cpu-seconds", "2")
+             "--cpu-seconds", "2", "--no-per-workload")
     _common(d)
     assert d["n_gpus"] == 1 and d["steps"] == 3 and d["warmup"] == 3
     assert d["dtype"] == "bf16"
@@ -85,3 +85,53 @@ def test_traffic_is_reported_only_for_the_profiled_source(tmp_path, monkeypatch)
     assert bench.load_traffic("missing_case") is None
     src.write_bytes(b"__global__ void k() { /* changed */ }\n")
     assert bench.load_traffic("k_case") is None
+
+
+@pytest.mark.gpu
+def test_per_workload_leg_keys():
+    """One per-workload leg (the tiny stream): the keys the bench line
+    carries for each stream of the metric."""
+    sys.path.insert(0, ROOT)
+    import torch
+    import bench
+    from paper_2609_36757_gb300 import workloads as WL
+    peaks, _ = bench.load_peaks()
+    leg = bench.measure_workload(WL.TINY, torch.device("cuda", 0), peaks, 0,
+                                 steps=2, warmup=1)
+    assert leg["steps"] == 2 and leg["warmup"] == 1
+    assert leg["flops_per_step"] > 0
+    for k in ("path_tflops", "kernel_tflops", "latent_frames_per_s",
+              "kernel_frac_of_sustained", "kernel_frac_of_burst"):
+        assert leg[k] > 0, k
+    assert leg["kernel_tflops"] >= leg["path_tflops"] * 0.5
+    assert set(leg["ms_per_chunk"]) == {"mean_fwd", "last_fwd",
+                                        "mean_step_per_chunk"}
+    assert leg["gpu_launches"] >= 2 * WL.TINY.num_chunks * 2
+    assert leg["shape"]["chunks"] == WL.TINY.num_chunks
+
+
+def test_append_dram_is_reported_only_for_the_profiled_source(tmp_path,
+                                                             monkeypatch):
+    """The append's DRAM-seen bytes come from a committed ncu summary only
+    while the append kernel source is unchanged (else null)."""
+    import hashlib
+    sys.path.insert(0, ROOT)
+    import bench
+    src = tmp_path / "paper_2609_36757_gb300" / "csrc" / "kv_append.cu"
+    src.parent.mkdir(parents=True)
+    src.write_bytes(b"// append\n")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    digest = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    (prof / "kv_append_1080p_traffic.txt").write_text(
+        "source=kv_append.cu\nsource_sha256_16=%s\n"
+        "algorithmic_read_bytes=100\nalgorithmic_write_bytes=100\n"
+        "dram_read_bytes=100\ndram_write_bytes_during_launch=40\n"
+        "ncu_time_ns=1000\n" % digest)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    d = bench.append_dram({"hbm_gbs": 1000.0})
+    assert d["read_bytes"] == 100 and d["write_bytes_during_launch"] == 40
+    assert abs(d["dram_gbs_during_launch"] - 140.0 / 1000e-9 / 1e9) < 1e-9
+    assert abs(d["dram_frac_of_hbm"] - d["dram_gbs_during_launch"] / 1000.0) < 1e-12
+    src.write_bytes(b"// changed\n")
+    assert bench.append_dram({"hbm_gbs": 1000.0}) is None
