@@ -12,23 +12,29 @@
 //   warp 8      TMA producer of the Q tiles (once) and the K ring (3 deep);
 //   warp 10     TMA producer of the V ring (2 deep); all tiles are
 //               128-byte swizzled boxes of 64 columns.
+//   warp 11     relay: observes the TMA completions and hands each K/V ring
+//               stage to the MMA warp through a named barrier.
 //   warp 9      MMA issuer (the warp runs converged, an elected lane
-//               issues): S_t = Q_t K^T into TMEM, then O_t += P_t V with
-//               P_t read from TMEM.
+//               issues): S = Q_t K^T into TMEM, then O_t += P_t V with P_t
+//               read from TMEM; order per key tile j: QK_0(j), PV_0(j-1),
+//               QK_1(j), PV_1(j-1).
 //   warps 0-3   softmax of query tile 0, one thread per row (TMEM lane);
 //   warps 4-7   softmax of query tile 1.
-// TMEM (512 columns): S_0 | S_1 | O_0 | O_1, 128 columns each; P_t (bf16
-// pairs, 64 columns) overwrites the first half of S_t once S_t is in
-// registers.  The two query tiles alternate on the tensor pipe, so one
-// tile's softmax overlaps the other tile's MMAs.
+// TMEM (512 columns): S (shared by the two tiles) | P_0 | P_1 | O_0 | O_1,
+// 128 + 64 + 64 + 128 + 128 columns.  S only lives until the softmax warps
+// have loaded it (they release it before the row max), so the next QK^T of
+// either tile can follow at once; each tile's PV runs one key tile behind,
+// which gives its softmax three MMA steps to store P_t.  The MMA warp never
+// polls a shared-memory barrier: every hand-off to it (S read, P_t stored,
+// K/V stage landed) is a named barrier, whose arrivals are made on every
+// path (also after a failed wait), since a named barrier has no time limit.
 //
 // Online softmax in the exp2 domain: each row keeps a reference m (a lower
 // bound of its running max) and exponentiates against it; m moves, and O is
 // rescaled, only when a tile's max exceeds m by more than 8 (P stays <= 256,
 // finite in bf16 and fp32).  The final O / l is the same for any reference,
-// so this is exact up to rounding.  When S_t(j) is ready, PV_t(j-1) has
-// completed too (one commit tracks every earlier MMA), so the rescale needs
-// no extra wait.
+// so this is exact up to rounding.  Before storing P_t(j) the softmax waits
+// until PV_t(j-1) has completed, so O_t is current for the rare rescale.
 //
 // Every mbarrier wait is bounded: past the limit the kernel records
 // FASTVR timeout in the control word, all roles stop issuing, in-flight TMA
