@@ -512,11 +512,16 @@ def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
     for i in range(args.warmup):
         step(evs[i])
     torch.cuda.synchronize(dev)
+    clocks = ClockSampler(local_rank) if rank == 0 else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
     barrier(world)
     for i in range(args.warmup, args.warmup + args.steps):
         step(evs[i])
     torch.cuda.synchronize(dev)
     barrier(world)
+    clock_info = clocks.stop() if clocks else None
     timed = evs[args.warmup:]
     fwd_ms = statistics.median(e[0].elapsed_time(e[1]) for e in timed)
     bwd_ms = statistics.median(e[1].elapsed_time(e[2]) for e in timed)
@@ -537,6 +542,7 @@ def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
                    "head_dim": w.head_dim, "tokens": w.num_tokens,
                    "frames_per_chunk": w.frames_per_chunk,
                    "window_chunks": w.window_chunks, "mode": args.mode},
+        "clocks": clock_info,
         "fwd_ms": fwd_ms, "fwd_tflops": fwd_flops / (fwd_ms / 1e3) / 1e12,
         "fwd_frac_of_burst_peak": fwd_flops / (fwd_ms / 1e3) / 1e12 /
                                   peaks["bf16_tflops"],

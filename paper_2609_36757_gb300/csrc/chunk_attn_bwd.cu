@@ -42,14 +42,14 @@ constexpr int kT = 128;           // tile rows (TMEM lanes) and tile columns
 constexpr int kBox = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (bytes)
 constexpr int kMaxStages = 3;     // deepest streamed ring
 constexpr int kStages1 = 2;       // ring 1 depth (ring 0: per kernel)
-constexpr int kDkdvS0 = 2;        // dK/dV ring 0 (Q and row vectors)
+constexpr int kDkdvS0 = 3;        // dK/dV ring 0 (Q)
 constexpr int kDqS0 = 3;          // dQ ring 0 (K): loads one step earlier
-static_assert(kDkdvS0 == kStages1, "dK/dV indexes both rings alike");
-constexpr int kThreads = 352;     // 8 compute warps, producer, MMA issuer,
-                                  // relay
+constexpr int kThreads = 384;     // 8 compute warps, producer, MMA issuer,
+                                  // relay, row-vector loader (dK/dV)
 constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kRelayWarp = 10;
+constexpr int kVecWarp = 11;
 // Named (hardware) barriers of the hand-offs to the MMA warp: P stored and
 // dS stored (the eight compute warps arrive, the MMA warp syncs), and one
 // per stage of each streamed ring (the relay warp arrives once the stage's
@@ -88,19 +88,23 @@ struct BwdShared {
   // reader has run instead of waiting for the end of the step.
   uint64_t full[2][kMaxStages], empty[2][kMaxStages];
   uint64_t s_ready, dp_ready, o_full, drain;
+  // dK/dV: the two slots of -log2 LSE and -D slices (loaded by the
+  // row-vector warp, released by the compute warps after dS)
+  uint64_t vec_full[2], vec_empty[2];
   uint32_t tmem_base;
   int abort;
   int* status;
   uint64_t wait_limit_ns;
 };
 
-// Shared memory: the two fixed operands, ring 0 (kS0 stages), ring 1
-// (kStages1 stages), the barriers, and with kVecs the per-stage slices of
-// -log2 LSE and -D for ring 0's query tiles (dK/dV).  The dQ kernel's third
-// K stage fits only because it carries no slices.
-template <int D, int kS0, bool kVecs>
+// Shared memory of the dQ kernel: the two fixed operands, ring 0 (kS0
+// stages), ring 1 (kStages1 stages), then the barriers; the dynamic base is
+// rounded up to 1024 bytes (128-byte-swizzled tiles), which the size allows
+// for.
+template <int D, int S0>
 struct BwdLayout {
-  static_assert(kS0 >= 2 && kS0 <= kMaxStages, "ring 0 depth");
+  static_assert(S0 >= 2 && S0 <= kMaxStages, "ring 0 depth");
+  static constexpr int kS0 = S0;
   static constexpr int kNB = D / 64;
   __host__ __device__ static constexpr int fixed(int which, int bx) {
     return (which * kNB + bx) * kBox;
@@ -109,15 +113,36 @@ struct BwdLayout {
     return ((2 + (which ? kS0 + st : st)) * kNB + bx) * kBox;
   }
   static constexpr int shared_off = (2 + kS0 + kStages1) * kNB * kBox;
-  static constexpr int vec_off =
-      shared_off + ((int)sizeof(BwdShared) + 15) / 16 * 16;
-  static constexpr int vec_bytes = kVecs ? 2 * kS0 * kT * (int)sizeof(float) : 0;
-  static constexpr int bytes = vec_off + vec_bytes + 1024 + 64;
-  // slice of stage st: lse2 at vec(0, st), dlt at vec(1, st) (floats)
-  __host__ __device__ static constexpr int vec(int which, int st) {
-    return vec_off + (which * kS0 + st) * kT * (int)sizeof(float);
-  }
+  static constexpr int bytes =
+      shared_off + ((int)sizeof(BwdShared) + 15) / 16 * 16 + 1024 + 64;
 };
+
+// Shared memory of the dK/dV kernel: a 3 KB front region (the barriers at 0,
+// the two slots of row vectors from 1024: slot sl holds 128 -log2 LSE values
+// then 128 -D values), then the two fixed operands, the three-stage Q ring
+// and the two-stage dO ring.  That is 227 KB exactly at d = 128, with no room
+// left to round the base up: the kernel requires (and checks) that the
+// dynamic shared memory starts 1024-byte aligned.
+template <int D>
+struct DkdvLayout {
+  static constexpr int kS0 = kDkdvS0;
+  static constexpr int kNB = D / 64;
+  static constexpr int kFrontBytes = 3072;
+  static constexpr int shared_off = 0;
+  __host__ __device__ static constexpr int vec(int slot, int which) {
+    return 1024 + (slot * 2 + which) * kT * (int)sizeof(float);
+  }
+  __host__ __device__ static constexpr int fixed(int which, int bx) {
+    return kFrontBytes + (which * kNB + bx) * kBox;
+  }
+  __host__ __device__ static constexpr int ring(int st, int which, int bx) {
+    return kFrontBytes + ((2 + (which ? kS0 + st : st)) * kNB + bx) * kBox;
+  }
+  static constexpr int bytes = kFrontBytes + (2 + kS0 + kStages1) * kNB * kBox;
+};
+static_assert(sizeof(BwdShared) <= 1024, "barriers fit the front region");
+static_assert(DkdvLayout<128>::vec(1, 1) + 128 * 4 <= DkdvLayout<128>::kFrontBytes,
+              "row-vector slots fit the front region");
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -256,6 +281,10 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S,
       }
     mbar_init(&S->s_ready, 1);
     mbar_init(&S->dp_ready, 1);
+    for (int sl = 0; sl < 2; ++sl) {
+      mbar_init(&S->vec_full[sl], 1);
+      mbar_init(&S->vec_empty[sl], 8);  // one arrival per compute warp
+    }
     mbar_init(&S->o_full, 1);
     mbar_init(&S->drain, 1);
     S->abort = 0;
@@ -280,16 +309,12 @@ __device__ __forceinline__ void bwd_teardown(uint32_t tmem) {
 
 // Producer: two resident tiles (maps f0, f1 at token t_fixed), then two
 // streamed tiles per step (maps r0, r1 at token t0 + 128 j).
-// With kRowVecs, each step also bulk-copies the streamed tile's 128 log2-LSE
-// and D values (from the padded scratch rows vec_lse2, vec_dlt).
-template <int D, bool kRowVecs, int kS0>
+template <class L>
 __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
                              const CUtensorMap* f1, int t_fixed,
                              const CUtensorMap* r0, const CUtensorMap* r1,
-                             int t0, int n, int h, int b,
-                             const float* vec_lse2, const float* vec_dlt) {
-  using L = BwdLayout<D, kS0, kRowVecs>;
-  constexpr uint32_t kVecBytes = kRowVecs ? 2 * kT * sizeof(float) : 0;
+                             int t0, int n, int h, int b) {
+  constexpr int kS0 = L::kS0;
   mbar_arrive_expect_tx(&S->fixed_full, 2 * L::kNB * kBox);
   for (int bx = 0; bx < L::kNB; ++bx) {
     tma_load_4d(f0, smem + L::fixed(0, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
@@ -308,16 +333,10 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
                   t0 + j * kT, h, b);
     ++issued[1];
     if (!wait_bar(&S->empty[0][s0], ((j / kS0) & 1) ^ 1, S)) break;
-    mbar_arrive_expect_tx(&S->full[0][s0], L::kNB * kBox + kVecBytes);
+    mbar_arrive_expect_tx(&S->full[0][s0], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
       tma_load_4d(r0, smem + L::ring(s0, 0, bx), &S->full[0][s0], bx * 64,
                   t0 + j * kT, h, b);
-    if (kRowVecs) {
-      bulk_load(smem + L::vec(0, s0), vec_lse2 + t0 + j * kT, kT * sizeof(float),
-                &S->full[0][s0]);
-      bulk_load(smem + L::vec(1, s0), vec_dlt + t0 + j * kT, kT * sizeof(float),
-                &S->full[0][s0]);
-    }
     ++issued[0];
   }
   drain_wait(&S->fixed_full, 0);
@@ -468,10 +487,17 @@ __device__ __forceinline__ void ds32(const uint32_t (&pb)[16],
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 dkdv_kernel(const __grid_constant__ BwdParams p) {
-  using L = BwdLayout<D, kDkdvS0, true>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  using L = DkdvLayout<D>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  // The layout fills 227 KB with no slack to round the base up: a base that
+  // is not 1024-byte aligned (which the 128-byte-swizzled tiles need) is
+  // reported as a failed bounds check and nothing is computed.
+  if ((smem_addr(smem) & 1023u) != 0) {
+    if (threadIdx.x == 0 && p.status != nullptr)
+      atomicExch(p.status, kDevBounds);
+    return;
+  }
   BwdShared* S = reinterpret_cast<BwdShared*>(smem + L::shared_off);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int bh = blockIdx.x % (p.heads * p.batch);
@@ -492,13 +518,31 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
 
   if (warp == kProducerWarp) {
     if (lane == 0)
-      bwd_producer<D, true, kDkdvS0>(smem, S, &p.k_map, &p.v_map, k0, &p.q_map,
-                            &p.do_map, q0, n, h, b,
-                            p.lse2 + (int64_t)bh_row(p, b, h) * p.padded,
-                            p.delta + (int64_t)bh_row(p, b, h) * p.padded);
+      bwd_producer<L>(smem, S, &p.k_map, &p.v_map, k0, &p.q_map, &p.do_map,
+                      q0, n, h, b);
     __syncwarp();
   } else if (warp == kRelayWarp) {
     bwd_relay<kDkdvS0>(S, n);
+  } else if (warp == kVecWarp) {
+    // Row vectors: step j's 128 -log2 LSE and -D values into slot j % 2,
+    // once the compute warps have released the slot (after dS of step j-2).
+    if (lane == 0) {
+      const int64_t row = (int64_t)bh_row(p, b, h) * p.padded;
+      int issued = 0;
+      for (int j = 0; j < n; ++j) {
+        const int sl = j & 1;
+        if (!wait_bar(&S->vec_empty[sl], ((j >> 1) & 1) ^ 1, S)) break;
+        mbar_arrive_expect_tx(&S->vec_full[sl], 2 * kT * sizeof(float));
+        bulk_load(smem + L::vec(sl, 0), p.lse2 + row + q0 + j * kT,
+                  kT * sizeof(float), &S->vec_full[sl]);
+        bulk_load(smem + L::vec(sl, 1), p.delta + row + q0 + j * kT,
+                  kT * sizeof(float), &S->vec_full[sl]);
+        ++issued;
+      }
+      for (int i = max(0, issued - 2); i < issued; ++i)
+        drain_wait(&S->vec_full[i & 1], (i >> 1) & 1);
+    }
+    __syncwarp();
   } else if (warp == kMmaWarp) {
     const uint32_t sbase = smem_addr(smem);
     // The next tile's S^T is issued right after this tile's dV (it
@@ -521,25 +565,27 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       mma_commit_warp(&S->dp_ready);
     }
     for (int j = 0; ok && j < n; ++j) {
-      const int st = j % kStages1, stn = (j + 1) % kStages1;
+      // Q (ring 0) and dO (ring 1) run at their own depths
+      const int q_st = j % kDkdvS0, q_stn = (j + 1) % kDkdvS0;
+      const int o_st = j % kStages1, o_stn = (j + 1) % kStages1;
       compute_sync(kBarP);
       tc_fence_after();
-      mma_tn<D>(sbase, tmem, 256, 0, L::ring(st, 1, 0), j > 0);    // dV
-      mma_commit_warp(&S->empty[1][st]);  // dO_j read for the last time
+      mma_tn<D>(sbase, tmem, 256, 0, L::ring(o_st, 1, 0), j > 0);    // dV
+      mma_commit_warp(&S->empty[1][o_st]);  // dO_j read for the last time
       if (j + 1 < n) {
-        relay_sync(kBarRing0 + stn);
+        relay_sync(kBarRing0 + q_stn);
         tc_fence_after();
-        mma_nt<D, L>(sbase, tmem, 0, 0, stn, 0);  // S^T_{j+1}
+        mma_nt<D, L>(sbase, tmem, 0, 0, q_stn, 0);  // S^T_{j+1}
         mma_commit_warp(&S->s_ready);
       }
       compute_sync(kBarDS);
       tc_fence_after();
-      mma_tn<D>(sbase, tmem, 384, 128, L::ring(st, 0, 0), j > 0);  // dK
-      mma_commit_warp(&S->empty[0][st]);  // Q_j and the row vectors
+      mma_tn<D>(sbase, tmem, 384, 128, L::ring(q_st, 0, 0), j > 0);  // dK
+      mma_commit_warp(&S->empty[0][q_st]);  // Q_j read for the last time
       if (j + 1 < n) {
-        relay_sync(kBarRing1 + stn);
+        relay_sync(kBarRing1 + o_stn);
         tc_fence_after();
-        mma_nt<D, L>(sbase, tmem, 128, 1, stn, 1);  // dP^T_{j+1}
+        mma_nt<D, L>(sbase, tmem, 128, 1, o_stn, 1);  // dP^T_{j+1}
         mma_commit_warp(&S->dp_ready);
       }
     }
@@ -563,13 +609,12 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     int p_arr = 0, ds_arr = 0;  // hand-offs made to the MMA warp
     for (int j = 0; j < n; ++j) {
       const int i0 = q0 + j * kT + 64 * hf;  // first query of this half
-      const int st = j % kDkdvS0;
-      // the stage's LSE and D slices (the MMA warp frees the stage only after
-      // ds_ready, so they stay valid while this tile is processed)
-      if (!(ok = wait_bar_warp(&S->full[0][st], (j / kDkdvS0) & 1, S))) break;
+      const int sl = j & 1;
+      // this step's LSE and D slices (released after dS, below)
+      if (!(ok = wait_bar_warp(&S->vec_full[sl], (j >> 1) & 1, S))) break;
       // -log2 LSE and -D per column
-      const float* nl = reinterpret_cast<const float*>(smem + L::vec(0, st)) + 64 * hf;
-      const float* nd = reinterpret_cast<const float*>(smem + L::vec(1, st)) + 64 * hf;
+      const float* nl = reinterpret_cast<const float*>(smem + L::vec(sl, 0)) + 64 * hf;
+      const float* nd = reinterpret_cast<const float*>(smem + L::vec(sl, 1)) + 64 * hf;
       // the first half's LSE values land while S^T is computed
       float4 la[8], lb[8];
 #pragma unroll
@@ -616,6 +661,9 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       tc_fence_before();
       compute_arrive(kBarDS);
       ++ds_arr;
+      // the row-vector slot is read for the last time
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S->vec_empty[sl]);
     }
     // After a failed wait the remaining hand-offs are still made (with
     // undefined contents), so that the MMA warp never waits for an arrival
@@ -647,7 +695,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 dq_kernel(const __grid_constant__ BwdParams p) {
-  using L = BwdLayout<D, kDqS0, false>;
+  using L = BwdLayout<D, kDqS0>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -666,11 +714,14 @@ dq_kernel(const __grid_constant__ BwdParams p) {
 
   if (warp == kProducerWarp) {
     if (lane == 0)
-      bwd_producer<D, false, kDqS0>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map,
-                             &p.v_map, kv0, n, h, b, nullptr, nullptr);
+      bwd_producer<L>(smem, S, &p.q_map, &p.do_map, q0, &p.k_map, &p.v_map,
+                      kv0, n, h, b);
     __syncwarp();
   } else if (warp == kRelayWarp) {
     bwd_relay<kDqS0>(S, n);
+  } else if (warp == kVecWarp) {
+    // no row-vector warp here: each compute thread reads its own row's two
+    // values once
   } else if (warp == kMmaWarp) {
     const uint32_t sbase = smem_addr(smem);
     // S of the next tile is issued as soon as P of this one is in
@@ -949,10 +1000,10 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   delta_kernel<D><<<(unsigned)blocks, 256, 0, stream>>>(
       a.out, a.dout, a.lse, a.scratch, a.scratch + (size_t)a.batch * a.heads * padded,
       a.batch, a.heads, L, padded);
-  const int smem = BwdLayout<D, kDkdvS0, true>::bytes;
-  const int smem_dq = BwdLayout<D, kDqS0, false>::bytes;
-  static_assert(BwdLayout<128, kDkdvS0, true>::bytes <= 227 * 1024 &&
-                    BwdLayout<128, kDqS0, false>::bytes <= 227 * 1024,
+  const int smem = DkdvLayout<D>::bytes;
+  const int smem_dq = BwdLayout<D, kDqS0>::bytes;
+  static_assert(DkdvLayout<128>::bytes <= 227 * 1024 &&
+                    BwdLayout<128, kDqS0>::bytes <= 227 * 1024,
                 "backward shared memory");
   cudaError_t e = cudaFuncSetAttribute(
       dkdv_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
