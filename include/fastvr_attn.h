@@ -63,8 +63,9 @@ typedef enum {
                                   ragged (final) chunk                        */
   FASTVR_ERR_CUDA = 5,         /* a CUDA runtime/driver call failed           */
   FASTVR_ERR_TIMEOUT = 6,      /* a bounded device-side wait gave up          */
-  FASTVR_ERR_BOUNDS = 7        /* debug library only: a device-side index
-                                  check failed and the access was skipped     */
+  FASTVR_ERR_BOUNDS = 7        /* a device-side index or layout check failed
+                                  and the access was skipped (index checks:
+                                  debug library only)                        */
 } fastvr_status_t;
 
 typedef struct {
@@ -196,7 +197,10 @@ FASTVR_API fastvr_status_t fastvr_blockcausal_bwd_scratch_bytes(
  * tiles that see them) and dq (one CTA per 128 queries); P is recomputed
  * from lse, P and dS enter the tensor cores in bfloat16, accumulation is
  * fp32.  All pointers 16-byte aligned.  A bounded-wait timeout leaves the
- * outputs undefined and is reported by fastvr_get_device_status.
+ * outputs undefined and is reported by fastvr_get_device_status
+ * (FASTVR_ERR_TIMEOUT); so is a dynamic shared-memory base that is not
+ * 1024-byte aligned, which the dK/dV kernel's 227 KB layout requires and
+ * checks (FASTVR_ERR_BOUNDS, nothing computed).
  * Errors: INVALID_ARG, UNSUPPORTED, CAPACITY (scratch too small), CUDA. */
 FASTVR_API fastvr_status_t fastvr_blockcausal_attn_bwd(
     const fastvr_attn_config_t* cfg, int32_t num_frames, const void* q,

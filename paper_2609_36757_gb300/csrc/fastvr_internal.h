@@ -37,7 +37,8 @@ EncodeTiledFn encode_tiled_fn();
 // Error codes a kernel writes into the cache's control block.
 constexpr int kDevOk = 0;
 constexpr int kDevTimeout = 1;
-constexpr int kDevBounds = 2;  // debug builds: an index check failed
+constexpr int kDevBounds = 2;  // an index check (debug builds) or a layout
+                               // check failed
 
 #ifdef __CUDACC__
 // Debug builds (-DFASTVR_BOUNDS_CHECK, libfastvr_attn_debug.so) check every
