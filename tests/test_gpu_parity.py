@@ -200,3 +200,68 @@ def test_paper_tiles_32x32_sampled_rows():
 
 def test_paper_tiles_64x64_sampled_rows():
     run_stream(WL.PAPER_TILES_64, rows_per_chunk=256).check()
+
+
+# ------------------------------------ dependencies on the previous work
+# The library's kernels start with programmatic dependent launch and wait
+# for the preceding kernel before touching its data.  These streams feed
+# every call from work queued just before it, with no synchronisation in
+# between: (a) torch kernels on the same stream that produce q, k and v, and
+# (b) pinned-host copies on a side stream that the compute stream waits for
+# through events (the pattern of an end-to-end pipeline).
+def test_inputs_from_kernels_queued_just_before():
+    w = SMALL[1]
+    from paper_2609_36757_gb300 import fastvr as FV
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    outs = []
+    qs, ks, vs = [], [], []
+    for c, q, k, v in WL.chunk_stream(w):
+        qd, kd, vd = (x.cuda() for x in (q, k, v))
+        torch.cuda.synchronize()
+        # each input is rewritten by an elementwise kernel right before use
+        k2, v2, q2 = kd * 1.0, vd * 1.0, qd * 1.0
+        att.append(k2, v2)
+        o = att.forward(q2)
+        outs.append(o)
+        qs.append(q), ks.append(k), vs.append(v)
+    torch.cuda.synchronize()
+    ref_o, _ = OA.blockcausal_attention(
+        to64(torch.cat(qs, 1)), to64(torch.cat(ks, 1)), to64(torch.cat(vs, 1)),
+        w.tokens_per_frame, w.frames_per_chunk, w.window_chunks,
+        w.softmax_scale)
+    err = Err()
+    err.add(to64(torch.cat([o.cpu() for o in outs], 1)), ref_o)
+    err.check()
+    assert att.status() == FV.FASTVR_OK
+
+
+def test_inputs_from_side_stream_copies():
+    w = SMALL[0]
+    from paper_2609_36757_gb300 import fastvr as FV
+    att = FV.StreamingAttention(FV.config_from_workload(w))
+    compute = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    host = [(q.pin_memory(), k.pin_memory(), v.pin_memory())
+            for _, q, k, v in WL.chunk_stream(w)]
+    outs = []
+    for q, k, v in host:
+        with torch.cuda.stream(side):
+            qd, kd, vd = (x.to("cuda", non_blocking=True) for x in (q, k, v))
+            ready = torch.cuda.Event()
+            ready.record(side)
+        compute.wait_event(ready)
+        for x in (qd, kd, vd):
+            x.record_stream(compute)
+        att.append(kd, vd)
+        outs.append(att.forward(qd))
+    torch.cuda.synchronize()
+    ref_o, _ = OA.blockcausal_attention(
+        to64(torch.cat([h[0] for h in host], 1)),
+        to64(torch.cat([h[1] for h in host], 1)),
+        to64(torch.cat([h[2] for h in host], 1)),
+        w.tokens_per_frame, w.frames_per_chunk, w.window_chunks,
+        w.softmax_scale)
+    err = Err()
+    err.add(to64(torch.cat([o.cpu() for o in outs], 1)), ref_o)
+    err.check()
+    assert att.status() == FV.FASTVR_OK

@@ -103,3 +103,29 @@ def test_gpu_step_with_target_velocity_lands_on_hq():
     # only the rounding of u to bf16 separates the result from z_HQ
     bound = (sigma * (u.float() - (z_lq - z_hq) / sigma)).abs() + 1e-6
     assert ((out - z_hq).abs() <= bound * 1.0001 + 1e-6).all()
+
+
+@pytest.mark.gpu
+def test_gpu_chained_updates_on_the_same_stream():
+    """Back-to-back launches with no synchronisation: each update reads what
+    the kernel queued just before it wrote (the launches overlap their
+    set-up with the previous kernel's drain and must still wait for its
+    data)."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    n = 48 * 3 * 68 * 120 + 3
+    g = torch.Generator().manual_seed(6)
+    z = torch.randn(n, generator=g)
+    vs = [torch.randn(n, generator=g).to(torch.bfloat16) for _ in range(4)]
+    zd = z.cuda()
+    vd = [v.cuda() for v in vs]
+    torch.cuda.synchronize()
+    sig = [0.5, 0.25, 0.75, 0.125]
+    for v, s in zip(vd, sig):
+        FV.one_step_update(zd, v, s, out=zd)   # in place, one after another
+        zd = zd * 1.0                           # a torch kernel in between
+    ref = z.double().numpy()
+    for v, s in zip(vs, sig):
+        ref = OS.one_step_update(ref.astype(np.float32).astype(np.float64),
+                                 v.double().numpy(), float(np.float32(s)))
+    got = zd.cpu().double().numpy()
+    assert np.abs(got - ref).max() <= 4 * 2.0 ** -23 * np.abs(ref).max() + 1e-6
