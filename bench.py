@@ -611,6 +611,10 @@ def run_e2e(args, w, chunks, att, dev, step_flops, world):
     for _ in range(max(1, args.warmup)):
         step()
     torch.cuda.synchronize(dev)
+    clocks = ClockSampler(dev.index) if dev.index is not None else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
     barrier(world)
     t0 = time.perf_counter()
     for _ in range(args.steps):
@@ -618,8 +622,10 @@ def run_e2e(args, w, chunks, att, dev, step_flops, world):
     torch.cuda.synchronize(dev)
     barrier(world)
     dt = reduce_max(time.perf_counter() - t0, world)
+    clock_info = clocks.stop() if clocks else None
     return {"value": world * step_flops * args.steps / dt / 1e12, "unit": UNIT,
-            "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h_bytes}
+            "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h_bytes,
+            "clocks": clock_info}
 
 
 # ------------------------------------------------------------- distributed
