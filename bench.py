@@ -611,7 +611,8 @@ def run_e2e(args, w, chunks, att, dev, step_flops, world):
     for _ in range(max(1, args.warmup)):
         step()
     torch.cuda.synchronize(dev)
-    clocks = ClockSampler(dev.index) if dev.index is not None else None
+    rank0 = int(os.environ.get("RANK", "0")) == 0
+    clocks = ClockSampler(dev.index) if rank0 and dev.index is not None else None
     if clocks:
         clocks.start()
         time.sleep(0.3)
