@@ -429,14 +429,18 @@ __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
 // P = 2^(s c2 - lse2) for 32 columns [c0, c0 + 32) of a half row, packed to
-// bf16 pairs; columns outside [lo, hi) are masked (p = 0).  nl holds -lse2
-// for the 32 columns, in registers: the dK/dV kernel reads its per-column
-// values from shared memory ahead of use, because the SMEM x SMEM MMAs that
-// run meanwhile take all of the shared-memory bandwidth and each read waits
-// behind them.
+// bf16 pairs; with kMask, columns outside [lo, hi) are masked (p = 0).  nl
+// holds -lse2 for the 32 columns, in registers: the dK/dV kernel reads its
+// per-column values from shared memory ahead of use, because the SMEM x SMEM
+// MMAs that run meanwhile take all of the shared-memory bandwidth and each
+// read waits behind them.  The mask is a template argument, and the callers
+// branch on a warp vote: a mask tested at run time inside the loop costs two
+// compares and a select per element on every tile (measured: twice the time
+// of the unmasked form), while only tiles that cross a chunk edge need it.
+template <bool kMask>
 __device__ __forceinline__ void p32(const uint32_t (&s)[32],
                                     const float4 (&nl)[8], int c0, int lo,
-                                    int hi, bool need_mask, uint64_t c2x2,
+                                    int hi, uint64_t c2x2,
                                     uint32_t (&pp)[16]) {
 #pragma unroll
   for (int q = 0; q < 8; ++q) {  // four columns at a time
@@ -446,7 +450,7 @@ __device__ __forceinline__ void p32(const uint32_t (&s)[32],
                     c2x2, f2(a.x, a.y)), x[0], x[1]);
     f2_split(f2_fma(f2(__uint_as_float(s[4 * q + 2]), __uint_as_float(s[4 * q + 3])),
                     c2x2, f2(a.z, a.w)), x[2], x[3]);
-    if (need_mask) {
+    if (kMask) {
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const int col = c0 + 4 * q + u;
@@ -622,7 +626,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       if (!(ok = wait_bar_warp(&S->s_ready, j & 1, S))) break;
       tc_fence_after();
       const int lo = vis_lo - i0, hi = vis_hi - i0;
-      const bool need_mask = lo > 0 || hi < 64;
+      const bool need_mask = __any_sync(0xffffffffu, lo > 0 || hi < 64);
       uint32_t x0[32], x1[32], pb0[16], pb1[16], pk[16];
       // phase 1: P^T over the first half of S^T (for the dV MMA) and in
       // registers (for dS: the next tile's S^T may overwrite it in TMEM as
@@ -633,9 +637,15 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       for (int q = 0; q < 8; ++q)
         lb[q] = reinterpret_cast<const float4*>(nl + 32)[q];
       tmem_wait_ld();
-      p32(x0, la, 0, lo, hi, need_mask, c2x2, pb0);
-      tmem_st16(row_t + cs, pb0);
-      p32(x1, lb, 32, lo, hi, need_mask, c2x2, pb1);
+      if (need_mask) {
+        p32<true>(x0, la, 0, lo, hi, c2x2, pb0);
+        tmem_st16(row_t + cs, pb0);
+        p32<true>(x1, lb, 32, lo, hi, c2x2, pb1);
+      } else {
+        p32<false>(x0, la, 0, lo, hi, c2x2, pb0);
+        tmem_st16(row_t + cs, pb0);
+        p32<false>(x1, lb, 32, lo, hi, c2x2, pb1);
+      }
       tmem_st16(row_t + cs + 16, pb1);
       tmem_wait_st();
       tc_fence_before();
@@ -798,7 +808,8 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tc_fence_after();
       const int lo = vis_lo - tok0;
       const int hi = vis_hi - tok0;
-      const bool need_mask = lo > 0 || hi < 64 || !in_range;
+      const bool need_mask =
+          __any_sync(0xffffffffu, lo > 0 || hi < 64 || !in_range);
       const int lo_m = in_range ? lo : 64, hi_m = in_range ? hi : 0;
       uint32_t x0[32], x1[32], pb0[16], pb1[16], pk[16];
       // phase 1 (overlaps the dP MMAs): P (bf16 pairs) in registers; S is
@@ -806,8 +817,13 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tmem_ld32(row_t + cs, x0);
       tmem_ld32(row_t + cs + 32, x1);
       tmem_wait_ld();
-      p32(x0, nl_v, 0, lo_m, hi_m, need_mask, c2x2, pb0);
-      p32(x1, nl_v, 32, lo_m, hi_m, need_mask, c2x2, pb1);
+      if (need_mask) {
+        p32<true>(x0, nl_v, 0, lo_m, hi_m, c2x2, pb0);
+        p32<true>(x1, nl_v, 32, lo_m, hi_m, c2x2, pb1);
+      } else {
+        p32<false>(x0, nl_v, 0, lo_m, hi_m, c2x2, pb0);
+        p32<false>(x1, nl_v, 32, lo_m, hi_m, c2x2, pb1);
+      }
       tc_fence_before();
       compute_arrive(kBarP);
       ++p_arr;
