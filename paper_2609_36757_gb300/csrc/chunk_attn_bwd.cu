@@ -87,7 +87,10 @@ struct BwdShared {
   // dO, last read by dV), so a ring-1 slot is refilled as soon as its last
   // reader has run instead of waiting for the end of the step.
   uint64_t full[2][kMaxStages], empty[2][kMaxStages];
-  uint64_t s_ready, dp_ready, o_full, drain;
+  // dp_ready[1]: the dQ kernel's second dP buffer (one barrier per buffer,
+  // so a barrier never completes a second phase before its waiters saw the
+  // first)
+  uint64_t s_ready, dp_ready[2], o_full, drain;
   // dK/dV: the two slots of -log2 LSE and -D slices (loaded by the
   // row-vector warp, released by the compute warps after dS)
   uint64_t vec_full[2], vec_empty[2];
@@ -280,7 +283,8 @@ __device__ __forceinline__ uint32_t bwd_setup(BwdShared* S,
         mbar_init(&S->empty[r][s], 1);
       }
     mbar_init(&S->s_ready, 1);
-    mbar_init(&S->dp_ready, 1);
+    mbar_init(&S->dp_ready[0], 1);
+    mbar_init(&S->dp_ready[1], 1);
     for (int sl = 0; sl < 2; ++sl) {
       mbar_init(&S->vec_full[sl], 1);
       mbar_init(&S->vec_empty[sl], 8);  // one arrival per compute warp
@@ -566,7 +570,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       relay_sync(kBarRing1);
       tc_fence_after();
       mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP^T_0 = V dO_0^T
-      mma_commit_warp(&S->dp_ready);
+      mma_commit_warp(&S->dp_ready[0]);
     }
     for (int j = 0; ok && j < n; ++j) {
       // Q (ring 0) and dO (ring 1) run at their own depths
@@ -590,7 +594,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
         relay_sync(kBarRing1 + o_stn);
         tc_fence_after();
         mma_nt<D, L>(sbase, tmem, 128, 1, o_stn, 1);  // dP^T_{j+1}
-        mma_commit_warp(&S->dp_ready);
+        mma_commit_warp(&S->dp_ready[0]);
       }
     }
     if (ok) mma_commit_warp(&S->o_full);
@@ -655,7 +659,7 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
       // half of dP^T; the D values are read ahead like the LSE values
 #pragma unroll
       for (int q = 0; q < 8; ++q) la[q] = reinterpret_cast<const float4*>(nd)[q];
-      if (!(ok = wait_bar_warp(&S->dp_ready, j & 1, S))) break;
+      if (!(ok = wait_bar_warp(&S->dp_ready[0], j & 1, S))) break;
       tc_fence_after();
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
@@ -699,9 +703,10 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
 }
 
 // --------------------------------------------------------------------- dQ
-// TMEM: [0,128) S, [128,256) dP then dS (bf16, first 64 columns),
-// [256,256+d) dQ.  Resident: Q (fixed 0), dO (fixed 1).  Streamed: K (ring
-// 0), V (ring 1).
+// TMEM: [0,128) S, [128,256) and [384,512) dP then dS (bf16, first 64
+// columns) for even and odd steps, [256,256+d) dQ.  Resident: Q (fixed 0),
+// dO (fixed 1).  Streamed: K (ring 0), V (ring 1).
+__device__ __forceinline__ int dq_dp_col(int j) { return (j & 1) ? 384 : 128; }
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 dq_kernel(const __grid_constant__ BwdParams p) {
@@ -734,8 +739,9 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     // values once
   } else if (warp == kMmaWarp) {
     const uint32_t sbase = smem_addr(smem);
-    // S of the next tile is issued as soon as P of this one is in
-    // registers, so it overlaps the dS computation.
+    // S and dP of the next tile are issued as soon as P of this one is in
+    // registers, so they overlap the dS computation; dP alternates between
+    // two buffers, so it need not wait for this tile's dQ to read dS.
     // Test hook: o_full receives no arrival before the end, so this wait
     // runs out and exercises the abort path.
     bool ok = (!p.inject_stall || wait_bar_warp(&S->o_full, 0, S)) &&
@@ -747,9 +753,9 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       mma_commit_warp(&S->s_ready);
       relay_sync(kBarRing1);
       tc_fence_after();
-      mma_nt<D, L>(sbase, tmem, 128, 1, 0, 1);  // dP_0 = dO V_0^T
-      mma_commit_warp(&S->dp_ready);
-      mma_commit_warp(&S->empty[1][0]);           // V_0 read for the last time
+      mma_nt<D, L>(sbase, tmem, dq_dp_col(0), 1, 0, 1);  // dP_0 = dO V_0^T
+      mma_commit_warp(&S->dp_ready[0]);
+      mma_commit_warp(&S->empty[1][0]);  // V_0 read for the last time
     }
     for (int j = 0; ok && j < n; ++j) {
       // K (ring 0) and V (ring 1) run at their own depths
@@ -761,18 +767,17 @@ dq_kernel(const __grid_constant__ BwdParams p) {
         tc_fence_after();
         mma_nt<D, L>(sbase, tmem, 0, 0, k_stn, 0);  // S_{j+1}
         mma_commit_warp(&S->s_ready);
+        // dP_{j+1} goes to the buffer that dQ_{j-1} (issued before) read
+        relay_sync(kBarRing1 + v_stn);
+        tc_fence_after();
+        mma_nt<D, L>(sbase, tmem, dq_dp_col(j + 1), 1, v_stn, 1);
+        mma_commit_warp(&S->dp_ready[(j + 1) & 1]);
+        mma_commit_warp(&S->empty[1][v_stn]);  // V_{j+1} read for the last time
       }
       compute_sync(kBarDS);
       tc_fence_after();
-      mma_tn<D>(sbase, tmem, 256, 128, L::ring(k_st, 0, 0), j > 0);  // dQ
+      mma_tn<D>(sbase, tmem, 256, dq_dp_col(j), L::ring(k_st, 0, 0), j > 0);  // dQ
       mma_commit_warp(&S->empty[0][k_st]);  // K_j read for the last time
-      if (j + 1 < n) {
-        relay_sync(kBarRing1 + v_stn);
-        tc_fence_after();
-        mma_nt<D, L>(sbase, tmem, 128, 1, v_stn, 1);  // dP_{j+1}
-        mma_commit_warp(&S->dp_ready);
-        mma_commit_warp(&S->empty[1][v_stn]);  // V_{j+1} read for the last time
-      }
     }
     if (ok) mma_commit_warp(&S->o_full);
     mma_commit_warp(&S->drain);
@@ -785,7 +790,7 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     const int hf = warp / 4;
     const int t = (warp % 4) * 32 + lane;
     const uint32_t row_t = tmem + ((uint32_t)((warp % 4) * 32) << 16);
-    const uint32_t cs = 64 * hf, cp = 128 + 64 * hf;
+    const uint32_t cs = 64 * hf;
     const int row = q0 + t;
     const bool in_range = row < p.seq_tokens;
     int vis_lo, vis_hi;
@@ -827,9 +832,11 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       tc_fence_before();
       compute_arrive(kBarP);
       ++p_arr;
-      // phase 2 (overlaps the next tile's S MMAs): dS over the dP columns
-      if (!(ok = wait_bar_warp(&S->dp_ready, j & 1, S))) break;
+      // phase 2 (overlaps the next tile's S and dP MMAs): dS over this
+      // step's dP buffer
+      if (!(ok = wait_bar_warp(&S->dp_ready[j & 1], (j >> 1) & 1, S))) break;
       tc_fence_after();
+      const uint32_t cp = dq_dp_col(j) + 64 * hf;
       tmem_ld32(row_t + cp, x0);
       tmem_ld32(row_t + cp + 32, x1);
       tmem_wait_ld();
