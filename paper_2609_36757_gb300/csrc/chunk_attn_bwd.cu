@@ -508,9 +508,12 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
   }
   BwdShared* S = reinterpret_cast<BwdShared*>(smem + L::shared_off);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int bh = blockIdx.x % (p.heads * p.batch);
+  // Head-major order: the CTAs resident at one time cover one or two
+  // (batch, head) rows, whose Q and dO tiles then stay in L2 for all of
+  // them; within a head, key tiles ascend (the longest query ranges first).
+  const int bh = blockIdx.x / p.tiles;
   const int h = bh % p.heads, b = bh / p.heads;
-  const int k0 = (blockIdx.x / (p.heads * p.batch)) * kT;  // first key
+  const int k0 = (blockIdx.x % p.tiles) * kT;  // first key
   // Queries that see any key of the tile: chunks c(k0) .. c(k_last) + W.
   const int k_last = min(k0 + kT, p.seq_tokens) - 1;
   // Query tiles start at a multiple of 128 at or below the first visible
@@ -716,10 +719,11 @@ dq_kernel(const __grid_constant__ BwdParams p) {
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   BwdShared* S = reinterpret_cast<BwdShared*>(smem + L::shared_off);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int bh = blockIdx.x % (p.heads * p.batch);
+  // Head-major order (the resident CTAs share their K and V tiles in L2);
+  // within a head, the longest key ranges first.
+  const int bh = blockIdx.x / p.tiles;
   const int h = bh % p.heads, b = bh / p.heads;
-  // longest key ranges first
-  const int q0 = (p.tiles - 1 - blockIdx.x / (p.heads * p.batch)) * kT;
+  const int q0 = (p.tiles - 1 - blockIdx.x % p.tiles) * kT;
   const int q_last = min(q0 + kT, p.seq_tokens) - 1;
   const int c_lo = q0 / p.chunk_tokens, c_hi = q_last / p.chunk_tokens;
   const int kv0 = p.window < 0 ? 0 : max(0, c_lo - p.window) * p.chunk_tokens;
