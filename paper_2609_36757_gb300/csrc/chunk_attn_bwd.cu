@@ -60,6 +60,7 @@ constexpr int kBarP = 1;
 constexpr int kBarDS = 2;
 constexpr int kBarRing0 = 3;  // + stage, up to kMaxStages
 constexpr int kBarRing1 = 6;  // + stage, up to kStages1
+constexpr int kBarStaged = 8;  // the compute warps' output tiles are staged
 constexpr int kComputeHandoff = 9 * 32;
 constexpr int kRelayHandoff = 2 * 32;
 constexpr uint32_t kTmemCols = 512;
@@ -67,6 +68,7 @@ constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
 struct BwdParams {
   CUtensorMap q_map, k_map, v_map, do_map;  // {d, L, H, B} token-major
+  CUtensorMap dq_map, dk_map, dv_map;       // the outputs, the same form
   const float* lse2;   // -(forward LSE in log2 units) [B*H, Lpad] (scratch)
   const float* delta;  // -D [B*H, Lpad] (scratch); padding tokens hold 0
   uint16_t* dq;        // bf16 [B, L, H, d]
@@ -203,6 +205,10 @@ __device__ __forceinline__ void compute_arrive(int id) {
 }
 __device__ __forceinline__ void compute_sync(int id) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kComputeHandoff) : "memory");
+}
+// All eight compute warps (256 threads), and no other warp.
+__device__ __forceinline__ void compute_only_sync(int id) {
+  asm volatile("bar.sync %0, 256;" ::"r"(id) : "memory");
 }
 __device__ __forceinline__ void relay_arrive(int id) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "n"(kRelayHandoff) : "memory");
@@ -387,23 +393,43 @@ __device__ __forceinline__ void mma_tn(uint32_t sbase, uint32_t tmem, int c0,
                 b_lo + (uint32_t)(kk * 2048 >> 4), hi, kIdesc, (acc | kk) != 0);
 }
 
-// Write 32 fp32 accumulator columns (scaled) of a TMEM row as bf16.
-__device__ __forceinline__ void store_row32(uint32_t taddr, float mul,
-                                            uint16_t* dst, bool ok) {
-  uint32_t r[32];
-  tmem_ld32(taddr, r);
+// Stage 32 fp32 accumulator columns [c0, c0 + 32) (scaled, as bf16) of TMEM
+// row r into the output tile in shared memory: [128 x 64] bf16 boxes of
+// 128-byte rows, 128-byte swizzled (16-byte chunk k of row r at chunk
+// k ^ (r % 8)), the form a tiled TMA store of the token-major map reads.
+// Rows leave in whole tiles (TMA stores) instead of one thread's 64 bytes at
+// a stride of H d elements.
+__device__ __forceinline__ void stage_row32(uint32_t taddr, float mul,
+                                            uint8_t* tile, int r, int c0) {
+  uint32_t v[32];
+  tmem_ld32(taddr, v);
   tmem_wait_ld();
   uint32_t pk[16];
 #pragma unroll
   for (int i = 0; i < 16; ++i)
-    pk[i] = pack_bf16(__uint_as_float(r[2 * i]) * mul,
-                      __uint_as_float(r[2 * i + 1]) * mul);
-  if (ok) {
-    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    pk[i] = pack_bf16(__uint_as_float(v[2 * i]) * mul,
+                      __uint_as_float(v[2 * i + 1]) * mul);
+  uint8_t* row = tile + (c0 / 64) * kBox + r * 128;
+  const int k0 = (c0 % 64) / 8;
 #pragma unroll
-    for (int v = 0; v < 4; ++v)
-      d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
-  }
+  for (int q = 0; q < 4; ++q)
+    *reinterpret_cast<uint4*>(row + (((k0 + q) ^ (r & 7)) << 4)) =
+        make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+}
+
+// After every compute thread staged its rows: one thread stores the staged
+// tiles (one per map, kNB boxes each, rows from token t0) and waits until the
+// writes are performed, so that the shared memory outlives the reads and the
+// grid's completion covers the writes.
+template <int kNB>
+__device__ __forceinline__ void store_staged(const CUtensorMap* const* maps,
+                                             uint8_t* const* tiles, int nmaps,
+                                             int t0, int h, int b) {
+  for (int m = 0; m < nmaps; ++m)
+    for (int bx = 0; bx < kNB; ++bx)
+      tma_store_4d(maps[m], tiles[m] + bx * kBox, bx * 64, t0, h, b);
+  bulk_commit_group();
+  bulk_wait_group0();
 }
 
 __device__ __forceinline__ uint64_t f2(float lo, float hi) {
@@ -687,19 +713,24 @@ dkdv_kernel(const __grid_constant__ BwdParams p) {
     // that does not come.
     for (; p_arr < n; ++p_arr) compute_arrive(kBarP);
     for (; ds_arr < n; ++ds_arr) compute_arrive(kBarDS);
+    // dV and dK are staged in the first two Q stages (free once o_full has
+    // completed: every MMA has read its operands) and leave as TMA stores;
+    // rows past the sequence fall outside the map and are not written.
+    uint8_t* const tiles[2] = {smem + L::ring(0, 0, 0), smem + L::ring(1, 0, 0)};
     if (ok && wait_bar_warp(&S->o_full, 0, S)) {
       tc_fence_after();
-      const int key = k0 + t;
-      const bool in_range = key < p.seq_tokens;
-      const int64_t off = (int64_t)b * p.seq_tokens * p.heads * D +
-                          (int64_t)(in_range ? key : 0) * p.heads * D +
-                          (int64_t)h * D;
 #pragma unroll 1
       for (int c = hf * D / 64; c < (hf + 1) * D / 64; ++c) {
-        store_row32(row_t + 256 + c * 32, 1.f, p.dv + off + c * 32, in_range);
-        store_row32(row_t + 384 + c * 32, p.scale, p.dk + off + c * 32,
-                    in_range);
+        stage_row32(row_t + 256 + c * 32, 1.f, tiles[0], t, c * 32);
+        stage_row32(row_t + 384 + c * 32, p.scale, tiles[1], t, c * 32);
       }
+      fence_proxy_async_smem();
+    }
+    compute_only_sync(kBarStaged);
+    if (warp == 0 && lane == 0 && ok &&
+        !*reinterpret_cast<volatile int*>(&S->abort)) {
+      const CUtensorMap* const maps[2] = {&p.dv_map, &p.dk_map};
+      store_staged<L::kNB>(maps, tiles, 2, k0, h, b);
     }
   }
   bwd_teardown(tmem);
@@ -858,15 +889,21 @@ dq_kernel(const __grid_constant__ BwdParams p) {
     // that does not come.
     for (; p_arr < n; ++p_arr) compute_arrive(kBarP);
     for (; ds_arr < n; ++ds_arr) compute_arrive(kBarDS);
+    // dQ is staged in the first K stage (free once o_full has completed)
+    // and leaves as TMA stores; rows past the sequence are not written.
+    uint8_t* const tiles[1] = {smem + L::ring(0, 0, 0)};
     if (ok && wait_bar_warp(&S->o_full, 0, S)) {
       tc_fence_after();
-      const int64_t off = (int64_t)b * p.seq_tokens * p.heads * D +
-                          (int64_t)(in_range ? row : 0) * p.heads * D +
-                          (int64_t)h * D;
 #pragma unroll 1
       for (int c = hf * D / 64; c < (hf + 1) * D / 64; ++c)
-        store_row32(row_t + 256 + c * 32, p.scale, p.dq + off + c * 32,
-                    in_range);
+        stage_row32(row_t + 256 + c * 32, p.scale, tiles[0], t, c * 32);
+      fence_proxy_async_smem();
+    }
+    compute_only_sync(kBarStaged);
+    if (warp == 0 && lane == 0 && ok &&
+        !*reinterpret_cast<volatile int*>(&S->abort)) {
+      const CUtensorMap* const maps[1] = {&p.dq_map};
+      store_staged<L::kNB>(maps, tiles, 1, q0, h, b);
     }
   }
   bwd_teardown(tmem);
@@ -997,7 +1034,10 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   if (!token_major_map(&p.q_map, a.q, D, L, a.heads, a.batch) ||
       !token_major_map(&p.k_map, a.k, D, L, a.heads, a.batch) ||
       !token_major_map(&p.v_map, a.v, D, L, a.heads, a.batch) ||
-      !token_major_map(&p.do_map, a.dout, D, L, a.heads, a.batch))
+      !token_major_map(&p.do_map, a.dout, D, L, a.heads, a.batch) ||
+      !token_major_map(&p.dq_map, a.dq, D, L, a.heads, a.batch) ||
+      !token_major_map(&p.dk_map, a.dk, D, L, a.heads, a.batch) ||
+      !token_major_map(&p.dv_map, a.dv, D, L, a.heads, a.batch))
     return cudaErrorInvalidValue;
   const int padded = (L + kT - 1) / kT * kT;
   p.lse2 = a.scratch;

@@ -81,6 +81,34 @@ __device__ __forceinline__ void tma_load_4d(const CUtensorMap* map, void* dst,
       : "memory");
 }
 
+// 4-D tiled store of one box from shared memory (the map's box and swizzle;
+// elements outside the tensor are not written), tracked by bulk groups.
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* map,
+                                             const void* src, int32_t c0,
+                                             int32_t c1, int32_t c2,
+                                             int32_t c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.global.shared::cta.tile.bulk_group "
+      "[%0, {%2, %3, %4, %5}], [%1];" ::"l"(reinterpret_cast<uint64_t>(map)),
+      "r"(smem_addr(src)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
+
+// Close the bulk group of this thread's earlier bulk stores, and wait until
+// every group is complete (its writes performed).
+__device__ __forceinline__ void bulk_commit_group() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_group0() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// Orders this thread's generic-proxy shared-memory writes before later
+// async-proxy (TMA) accesses.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // 1-D bulk copy global -> shared (16-byte aligned addresses, size a multiple
 // of 16), completing on `bar`.
 __device__ __forceinline__ void bulk_load(void* dst, const void* src,
