@@ -281,6 +281,8 @@ def run_gpu(args, rank: int, world: int, local_rank: int) -> None:
         per_workload = {name: measure_workload(WL.WORKLOADS[name], dev,
                                                peaks, local_rank)
                         for name in PER_WORKLOADS}
+        per_workload[TRAIN_LEG] = measure_train_leg(WL.WORKLOADS[TRAIN_LEG],
+                                                    dev, peaks, local_rank)
 
     if rank != 0:
         return
@@ -481,22 +483,17 @@ def measure_one_step(dev, sets: int = 8, rounds: int = 3):
             "l2": f"{sets} distinct latents rotated ({sets * 6 * n / 1e6:.0f} MB)"}
 
 
-def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
-    """One-shot (training) form over a whole sequence: forward, and in
-    `train` mode the backward too.  FLOPs: forward 4 B H d x visible pairs;
-    backward 2.5 x that (five products of the same size: S recomputed, dP,
-    dV, dQ, dK; the kernels compute two more to avoid atomics, not counted)."""
+def measure_oneshot(w, q, k, v, dev, steps: int, warmup: int, clock_index,
+                    world: int = 1, train: bool = True):
+    """Median CUDA-event times of the one-shot forward and (train) backward
+    over `steps` timed calls on resident inputs [B, L, H, d], after
+    `warmup` untimed ones, with the clocks sampled meanwhile.  dO is drawn
+    on the device from a generator seeded with the workload's seed."""
     from paper_2609_36757_gb300 import fastvr as FV
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    w = WORKLOAD
-    lk = visible_tokens_per_chunk(w)
-    fwd_flops = sum(chunk_flops(w, lk[c], c) for c in range(w.num_chunks))
-    chunks = host_chunks(w, seed_offset=rank)
-    q, k, v = (torch.cat([c[i] for c in chunks], 1).to(dev) for i in range(3))
-    do = torch.randn_like(q, dtype=torch.float32).to(torch.bfloat16)
+    g = torch.Generator(device=dev)
+    g.manual_seed(w.seed + 1)
+    do = torch.randn(q.shape, generator=g, device=dev).to(torch.bfloat16)
     cfg = FV.config_from_workload(w)
-    train = args.mode == "train"
     stream = torch.cuda.current_stream(dev)
 
     def step(ev):
@@ -508,23 +505,80 @@ def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
         ev[2].record(stream)
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)]
-           for _ in range(args.warmup + args.steps)]
-    for i in range(args.warmup):
+           for _ in range(warmup + steps)]
+    for i in range(warmup):
         step(evs[i])
     torch.cuda.synchronize(dev)
-    clocks = ClockSampler(local_rank) if rank == 0 else None
+    clocks = ClockSampler(clock_index) if clock_index is not None else None
     if clocks:
         clocks.start()
         time.sleep(0.3)
     barrier(world)
-    for i in range(args.warmup, args.warmup + args.steps):
+    for i in range(warmup, warmup + steps):
         step(evs[i])
     torch.cuda.synchronize(dev)
     barrier(world)
     clock_info = clocks.stop() if clocks else None
-    timed = evs[args.warmup:]
-    fwd_ms = statistics.median(e[0].elapsed_time(e[1]) for e in timed)
-    bwd_ms = statistics.median(e[1].elapsed_time(e[2]) for e in timed)
+    timed = evs[warmup:]
+    return {"fwd_ms": statistics.median(e[0].elapsed_time(e[1]) for e in timed),
+            "bwd_ms": statistics.median(e[1].elapsed_time(e[2]) for e in timed),
+            "clocks": clock_info}
+
+
+def oneshot_flops(w) -> float:
+    """Forward FLOPs of the one-shot form: 4 B H d x visible pairs."""
+    lk = visible_tokens_per_chunk(w)
+    return sum(chunk_flops(w, lk[c], c) for c in range(w.num_chunks))
+
+
+# The training form in the default line: forward + backward of the training
+# clip (one shot, Eq. 1 with W = 1).
+TRAIN_LEG = "train-1024-clip"
+
+
+def measure_train_leg(w, dev, peaks, clock_index, steps: int = 5,
+                      warmup: int = 3):
+    """Forward and backward TFLOP/s of the one-shot form on `w`, inputs drawn
+    on the device with the workload's recipe; the backward counted as 2.5 x
+    the forward FLOPs (the five products a backward needs)."""
+    data = [(q, k, v) for _, q, k, v in WL.chunk_stream(w, device=str(dev))]
+    q, k, v = (torch.cat([x[i] for x in data], 1) for i in range(3))
+    del data
+    t = measure_oneshot(w, q, k, v, dev, steps, warmup, clock_index)
+    del q, k, v
+    torch.cuda.empty_cache()
+    f = oneshot_flops(w)
+    fwd = f / (t["fwd_ms"] / 1e3) / 1e12
+    bwd = 2.5 * f / (t["bwd_ms"] / 1e3) / 1e12
+    return {
+        "steps": steps, "warmup": warmup,
+        "shape": {"batch": w.batch, "heads": w.heads, "head_dim": w.head_dim,
+                  "tokens": w.num_tokens, "frames_per_chunk": w.frames_per_chunk,
+                  "window_chunks": w.window_chunks},
+        "fwd_flops": f, "bwd_flops": 2.5 * f,
+        "fwd_ms": t["fwd_ms"], "bwd_ms": t["bwd_ms"],
+        "fwd_tflops": fwd, "bwd_tflops": bwd,
+        "fwd_frac_of_burst": fwd / peaks["bf16_tflops"],
+        "bwd_frac_of_burst": bwd / peaks["bf16_tflops"],
+        "clocks": t["clocks"],
+    }
+
+
+def run_oneshot(args, rank: int, world: int, local_rank: int) -> None:
+    """One-shot (training) form over a whole sequence: forward, and in
+    `train` mode the backward too.  FLOPs: forward 4 B H d x visible pairs;
+    backward 2.5 x that (five products of the same size: S recomputed, dP,
+    dV, dQ, dK; the kernels compute two more to avoid atomics, not counted)."""
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = WORKLOAD
+    fwd_flops = oneshot_flops(w)
+    chunks = host_chunks(w, seed_offset=rank)
+    q, k, v = (torch.cat([c[i] for c in chunks], 1).to(dev) for i in range(3))
+    train = args.mode == "train"
+    t = measure_oneshot(w, q, k, v, dev, args.steps, args.warmup,
+                        local_rank if rank == 0 else None, world, train)
+    fwd_ms, bwd_ms, clock_info = t["fwd_ms"], t["bwd_ms"], t["clocks"]
     step_ms = reduce_max(fwd_ms + bwd_ms, world)
     if rank != 0:
         return

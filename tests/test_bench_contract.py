@@ -135,3 +135,26 @@ def test_append_dram_is_reported_only_for_the_profiled_source(tmp_path,
     assert abs(d["dram_frac_of_hbm"] - d["dram_gbs_during_launch"] / 1000.0) < 1e-12
     src.write_bytes(b"// changed\n")
     assert bench.append_dram({"hbm_gbs": 1000.0}) is None
+
+
+@pytest.mark.gpu
+def test_train_leg_keys():
+    """The training-form leg of the default line (forward + backward of one
+    one-shot sequence), on a small d = 128 sequence: keys and consistency of
+    the rates with the times."""
+    sys.path.insert(0, ROOT)
+    import torch
+    import bench
+    from paper_2609_36757_gb300 import workloads as WL
+    peaks, _ = bench.load_peaks()
+    w = WL.Workload("train-small", 1, 4, 128, 256, 2, 3, window_chunks=1,
+                    seed=11)
+    leg = bench.measure_train_leg(w, torch.device("cuda", 0), peaks, 0,
+                                  steps=2, warmup=1)
+    assert leg["steps"] == 2 and leg["warmup"] == 1
+    assert leg["bwd_flops"] == 2.5 * leg["fwd_flops"] > 0
+    for k in ("fwd_ms", "bwd_ms", "fwd_tflops", "bwd_tflops",
+              "fwd_frac_of_burst", "bwd_frac_of_burst"):
+        assert leg[k] > 0, k
+    assert abs(leg["bwd_tflops"] - leg["bwd_flops"] / leg["bwd_ms"] / 1e9) < 1e-6 * leg["bwd_tflops"]
+    assert leg["shape"]["tokens"] == w.num_tokens
