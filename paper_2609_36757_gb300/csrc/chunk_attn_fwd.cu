@@ -81,9 +81,13 @@ constexpr int kHandoff = 5 * 32;
 constexpr int kBarKFull0 = 4;  // + stage (kKStages of them)
 constexpr int kBarVFull0 = 7;  // + stage (kVStages of them)
 constexpr int kRelay = 2 * 32;
+// Named barrier of a query tile's four softmax warps: their rows of O are
+// staged for the tile's TMA store.
+constexpr int kBarOStaged0 = 9;  // + t
 
 struct TcParams {
   CUtensorMap q_map;                  // {d, Lq, H, B}
+  CUtensorMap o_map;                  // the output, the same form as q_map
   CUtensorMap k_map[kMaxSegments];    // {d, segment end, H, B} of the cache
   CUtensorMap v_map[kMaxSegments];
   uint16_t* o;
@@ -341,6 +345,10 @@ __device__ __forceinline__ void named_sync(int id) {
 }
 __device__ __forceinline__ void relay_arrive(int id) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "n"(kRelay) : "memory");
+}
+// The four softmax warps of one query tile (128 threads), and no other warp.
+__device__ __forceinline__ void tile_sync(int id) {
+  asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory");
 }
 __device__ __forceinline__ void relay_sync(int id) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(kRelay) : "memory");
@@ -688,8 +696,7 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
     named_arrive(kBarPFull0 + t);
     ++p_arrived;
   }
-  if (!ok || !wait_bar(&S->o_full, 0, S, p.status)) return;
-  tc_fence_after();
+  const bool have = ok && wait_bar(&S->o_full, 0, S, p.status);
   const Work w = cta_work<kOneShot>(p);
   const int r_unit = t * kBM + wq * 32 + lane;  // row within the unit
   const int row = w.q0 + r_unit;
@@ -697,6 +704,8 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   if (w.part >= 0) {
     // Partial result of a key range: O / l in fp32 (transposed, so a warp's
     // stores are contiguous) and the log2-domain log-sum-exp.
+    if (!have) return;
+    tc_fence_after();
     float* ws_o = p.ws + (size_t)w.part * D * kUnitRows;
     float* ws_l = p.ws_lse + (size_t)w.part * kUnitRows;
 #pragma unroll
@@ -717,30 +726,46 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
       ws_l[r_unit] = m_ref + __log2f(l);
     return;
   }
-  const bool in_range = row < p.q_tokens;
-  uint16_t* orow = p.o + (int64_t)w.b * p.o_str.batch +
-                   (int64_t)(in_range ? row : 0) * p.o_str.token +
-                   (int64_t)w.h * p.o_str.head;
+  // Whole unit: the tile's rows of O / l, as bf16, are staged in its Q tile
+  // (free: every MMA has completed) as 128-byte-swizzled [128 x 64] boxes,
+  // and leave as TMA tile stores (rows past the chunk fall outside the map
+  // and are not written), instead of each thread writing 16-byte pieces of
+  // its row at a stride of H d elements.  Every thread of the tile reaches
+  // the barrier, also after a failed wait.
+  uint8_t* tile = reinterpret_cast<uint8_t*>(S) - Layout<D>::shared_off +
+                  Layout<D>::q(t, 0);
+  const int rt = wq * 32 + lane;  // row within the tile
+  if (have) {
+    tc_fence_after();
 #pragma unroll
-  for (int c = 0; c < D / 32; ++c) {
-    uint32_t r[32];
-    tmem_ld32(tO + c * 32, r);
-    tmem_wait_ld();
-    uint32_t pk[16];
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t r[32];
+      tmem_ld32(tO + c * 32, r);
+      tmem_wait_ld();
+      uint32_t pk[16];
 #pragma unroll
-    for (int i = 0; i < 16; ++i)
-      pk[i] = pack_bf16(__uint_as_float(r[2 * i]) * inv_l,
-                        __uint_as_float(r[2 * i + 1]) * inv_l);
-    if (in_range) {
-      uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+      for (int i = 0; i < 16; ++i)
+        pk[i] = pack_bf16(__uint_as_float(r[2 * i]) * inv_l,
+                          __uint_as_float(r[2 * i + 1]) * inv_l);
+      uint8_t* line = tile + (c / 2) * kBox + rt * 128;
 #pragma unroll
-      for (int v = 0; v < 4; ++v)
-        if (in_bounds(orow - p.o + c * 32 + 8 * v, p.o_elems - 7, p.status))
-          dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+      for (int q = 0; q < 4; ++q)
+        *reinterpret_cast<uint4*>(line + ((((c % 2) * 4 + q) ^ (rt & 7)) << 4)) =
+            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
     }
+    fence_proxy_async_smem();
+  }
+  tile_sync(kBarOStaged0 + t);
+  if (wq == 0 && lane == 0 && have &&
+      !*reinterpret_cast<volatile int*>(&S->abort)) {
+    for (int bx = 0; bx < Layout<D>::kNB; ++bx)
+      tma_store_4d(&p.o_map, tile + bx * kBox, bx * 64, w.q0 + t * kBM, w.h,
+                   w.b);
+    bulk_commit_group();
+    bulk_wait_group0();
   }
   const int64_t lse_i = ((int64_t)w.b * p.heads + w.h) * p.q_tokens + row;
-  if (p.lse != nullptr && in_range &&
+  if (have && p.lse != nullptr && row < p.q_tokens &&
       in_bounds(lse_i, (int64_t)p.batch * p.heads * p.q_tokens, p.status))
     p.lse[lse_i] = (m_ref + __log2f(l)) * 0.6931471805599453f;
 }
@@ -969,6 +994,8 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
   memset(&p, 0, sizeof(p));
   const int64_t es = 2;  // bytes per bf16
   if (!make_map(&p.q_map, a.q, D, a.q_tokens, a.heads, a.batch,
+                a.q_str.token * es, a.q_str.head * es, a.q_str.batch * es) ||
+      !make_map(&p.o_map, a.o, D, a.q_tokens, a.heads, a.batch,
                 a.q_str.token * es, a.q_str.head * es, a.q_str.batch * es))
     return cudaErrorInvalidValue;
   int tiles = 0;
@@ -1041,6 +1068,8 @@ cudaError_t launch_oneshot_d(const OneShotParams& a, cudaStream_t stream) {
       !make_map(&p.k_map[0], a.k, D, a.seq_tokens, a.heads, a.batch, tok * es,
                 D * es, bat * es) ||
       !make_map(&p.v_map[0], a.v, D, a.seq_tokens, a.heads, a.batch, tok * es,
+                D * es, bat * es) ||
+      !make_map(&p.o_map, a.o, D, a.seq_tokens, a.heads, a.batch, tok * es,
                 D * es, bat * es))
     return cudaErrorInvalidValue;
   p.k_map[1] = p.k_map[0];
