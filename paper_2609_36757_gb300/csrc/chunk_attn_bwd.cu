@@ -913,67 +913,62 @@ dq_kernel(const __grid_constant__ BwdParams p) {
 // minus the forward LSE in log2 units (negated so that both enter packed
 // FMAs as addends), each [B*H, Lpad] with Lpad = L rounded up to 128 and
 // zeros in the padding (so every 128-token slice is aligned and in bounds).
-// D / 8 lanes per (b, token, head) row of O (one 16-byte piece each), so a
-// warp reads 32 / (D / 8) adjacent rows per instruction, and each lane keeps
-// kDeltaUnroll such row groups in flight.
-constexpr int kDeltaUnroll = 4;
+// A block takes kDeltaTokens tokens of one (batch, head): D / 8 lanes per
+// token row of O and dO (one 16-byte piece each; a row is 2 D contiguous
+// bytes), every load of the block issued before the first product, then the
+// block writes its kDeltaTokens values of -D and -log2 LSE as one contiguous
+// run each (through shared memory), and reads the forward LSE the same way.
+// Tokens past the sequence (up to the padded length) get zeros.
+constexpr int kDeltaTokens = 64;
+constexpr int kDeltaThreads = 256;
 
 template <int D>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(kDeltaThreads)
 delta_kernel(const uint16_t* o, const uint16_t* dO, const float* lse,
-             float* lse2, float* delta, int batch, int heads, int seq,
-             int padded) {
+             float* lse2, float* delta, int heads, int seq, int padded) {
   constexpr int kLanesPerRow = D / 8;
-  constexpr int kRowsPerWarp = 32 / kLanesPerRow;
-  const int64_t rows = (int64_t)batch * seq * heads;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
-  const int lane = threadIdx.x % 32;
-  const int sub = lane / kLanesPerRow, piece = lane % kLanesPerRow;
-  const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
-  const int64_t step = nwarps * kRowsPerWarp;  // rows between a lane's groups
-  for (int64_t r0 = warp * kRowsPerWarp; r0 < rows; r0 += step * kDeltaUnroll) {
-    uint4 a[kDeltaUnroll], g[kDeltaUnroll];
+  constexpr int kRowsPerPass = kDeltaThreads / kLanesPerRow;
+  constexpr int kPasses = kDeltaTokens / kRowsPerPass;
+  __shared__ float red[kDeltaTokens];
+  const int tiles = padded / kDeltaTokens;
+  const int bh = blockIdx.x / tiles;  // b * heads + h
+  const int t0 = (blockIdx.x % tiles) * kDeltaTokens;
+  const int b = bh / heads, h = bh % heads;
+  const int sub = threadIdx.x / kLanesPerRow, piece = threadIdx.x % kLanesPerRow;
+  uint4 a[kPasses], g[kPasses];
 #pragma unroll
-    for (int u = 0; u < kDeltaUnroll; ++u) {
-      const int64_t r = r0 + u * step + sub;  // r = (b, token, head)
-      a[u] = g[u] = make_uint4(0, 0, 0, 0);
-      if (r < rows) {
-        a[u] = __ldcs(reinterpret_cast<const uint4*>(o + r * D) + piece);
-        g[u] = __ldcs(reinterpret_cast<const uint4*>(dO + r * D) + piece);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kDeltaUnroll; ++u) {
-      const uint32_t* ap = reinterpret_cast<const uint32_t*>(&a[u]);
-      const uint32_t* gp = reinterpret_cast<const uint32_t*>(&g[u]);
-      float acc = 0.f;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        acc = fmaf(__uint_as_float(ap[e] << 16), __uint_as_float(gp[e] << 16), acc);
-        acc = fmaf(__uint_as_float(ap[e] & 0xffff0000u),
-                   __uint_as_float(gp[e] & 0xffff0000u), acc);
-      }
-#pragma unroll
-      for (int m = kLanesPerRow / 2; m > 0; m >>= 1)
-        acc += __shfl_xor_sync(0xffffffffu, acc, m);
-      const int64_t r = r0 + u * step + sub;
-      if (piece == 0 && r < rows) {
-        const int64_t h = r % heads, bt = r / heads;
-        const int64_t tok = bt % seq, b = bt / seq;
-        const int64_t i = (b * heads + h) * padded + tok;
-        delta[i] = -acc;
-        lse2[i] = -lse[(b * heads + h) * seq + tok] * 1.4426950408889634f;
-      }
+  for (int u = 0; u < kPasses; ++u) {
+    const int tok = t0 + u * kRowsPerPass + sub;
+    a[u] = g[u] = make_uint4(0, 0, 0, 0);
+    if (tok < seq) {
+      const int64_t r = ((int64_t)b * seq + tok) * heads + h;  // [B, L, H] row
+      a[u] = __ldcs(reinterpret_cast<const uint4*>(o + r * D) + piece);
+      g[u] = __ldcs(reinterpret_cast<const uint4*>(dO + r * D) + piece);
     }
   }
-  // padding tokens
-  const int64_t pad = padded - seq;
-  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  for (int64_t i = tid; i < (int64_t)batch * heads * pad;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t j = (i / pad) * padded + seq + i % pad;
-    delta[j] = 0.f;
-    lse2[j] = 0.f;
+#pragma unroll
+  for (int u = 0; u < kPasses; ++u) {
+    const uint32_t* ap = reinterpret_cast<const uint32_t*>(&a[u]);
+    const uint32_t* gp = reinterpret_cast<const uint32_t*>(&g[u]);
+    float acc = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      acc = fmaf(__uint_as_float(ap[e] << 16), __uint_as_float(gp[e] << 16), acc);
+      acc = fmaf(__uint_as_float(ap[e] & 0xffff0000u),
+                 __uint_as_float(gp[e] & 0xffff0000u), acc);
+    }
+#pragma unroll
+    for (int m = kLanesPerRow / 2; m > 0; m >>= 1)
+      acc += __shfl_xor_sync(0xffffffffu, acc, m);
+    if (piece == 0) red[u * kRowsPerPass + sub] = acc;
+  }
+  __syncthreads();
+  if (threadIdx.x < kDeltaTokens) {
+    const int tok = t0 + threadIdx.x;
+    const int64_t i = (int64_t)bh * padded + tok;
+    const bool in = tok < seq;
+    delta[i] = in ? -red[threadIdx.x] : 0.f;
+    lse2[i] = in ? -lse[(int64_t)bh * seq + tok] * 1.4426950408889634f : 0.f;
   }
 }
 
@@ -1061,12 +1056,11 @@ cudaError_t launch_bwd_d(const BwdArgs& a, cudaStream_t stream) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t rows = (int64_t)a.batch * L * a.heads;
-  int64_t blocks = std::min<int64_t>((int64_t)(sms > 0 ? sms : 152) * 8,
-                                     (rows + 7) / 8);
-  delta_kernel<D><<<(unsigned)blocks, 256, 0, stream>>>(
+  const int64_t blocks =
+      (int64_t)a.batch * a.heads * (padded / kDeltaTokens);
+  delta_kernel<D><<<(unsigned)blocks, kDeltaThreads, 0, stream>>>(
       a.out, a.dout, a.lse, a.scratch, a.scratch + (size_t)a.batch * a.heads * padded,
-      a.batch, a.heads, L, padded);
+      a.heads, L, padded);
   const int smem = DkdvLayout<D>::bytes;
   const int smem_dq = BwdLayout<D, kDqS0>::bytes;
   static_assert(DkdvLayout<128>::bytes <= 227 * 1024 &&
