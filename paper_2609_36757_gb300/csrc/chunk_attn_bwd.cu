@@ -325,10 +325,15 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
                              const CUtensorMap* r0, const CUtensorMap* r1,
                              int t0, int n, int h, int b) {
   constexpr int kS0 = L::kS0;
+  // The resident tiles are read by this CTA alone (evict first); the
+  // streamed tiles of a head are read by every CTA of the head (evict last).
+  const uint64_t once = l2_policy_evict_first(), keep = l2_policy_evict_last();
   mbar_arrive_expect_tx(&S->fixed_full, 2 * L::kNB * kBox);
   for (int bx = 0; bx < L::kNB; ++bx) {
-    tma_load_4d(f0, smem + L::fixed(0, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
-    tma_load_4d(f1, smem + L::fixed(1, bx), &S->fixed_full, bx * 64, t_fixed, h, b);
+    tma_load_4d_hint(f0, smem + L::fixed(0, bx), &S->fixed_full, bx * 64,
+                     t_fixed, h, b, once);
+    tma_load_4d_hint(f1, smem + L::fixed(1, bx), &S->fixed_full, bx * 64,
+                     t_fixed, h, b, once);
   }
   // Ring 1 first: its slot frees earlier in a step (after dP or dV), so its
   // next tile loads while the step still runs; ring 0 (after dQ or dK)
@@ -339,14 +344,14 @@ __device__ void bwd_producer(uint8_t* smem, BwdShared* S, const CUtensorMap* f0,
     if (!wait_bar(&S->empty[1][s1], ((j / kStages1) & 1) ^ 1, S)) break;
     mbar_arrive_expect_tx(&S->full[1][s1], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(r1, smem + L::ring(s1, 1, bx), &S->full[1][s1], bx * 64,
-                  t0 + j * kT, h, b);
+      tma_load_4d_hint(r1, smem + L::ring(s1, 1, bx), &S->full[1][s1],
+                       bx * 64, t0 + j * kT, h, b, keep);
     ++issued[1];
     if (!wait_bar(&S->empty[0][s0], ((j / kS0) & 1) ^ 1, S)) break;
     mbar_arrive_expect_tx(&S->full[0][s0], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(r0, smem + L::ring(s0, 0, bx), &S->full[0][s0], bx * 64,
-                  t0 + j * kT, h, b);
+      tma_load_4d_hint(r0, smem + L::ring(s0, 0, bx), &S->full[0][s0],
+                       bx * 64, t0 + j * kT, h, b, keep);
     ++issued[0];
   }
   drain_wait(&S->fixed_full, 0);

@@ -272,13 +272,17 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
   constexpr int kStages = kIsK ? kKStages : kVStages;
   uint64_t* full = kIsK ? S->k_full : S->v_full;
   uint64_t* empty = kIsK ? S->k_empty : S->v_empty;
+  // The query tiles are read by this CTA alone (evict first); the K and V
+  // tiles of a head are read by every unit of the head (evict last).
+  const uint64_t keep = l2_policy_evict_last();
   if (kIsK) {
     tma_prefetch_desc(&p.q_map);
+    const uint64_t once = l2_policy_evict_first();
     mbar_arrive_expect_tx(&S->q_full, w.nqt * L::kNB * kBox);
     for (int t = 0; t < w.nqt; ++t)
       for (int bx = 0; bx < L::kNB; ++bx)
-        tma_load_4d(&p.q_map, smem + L::q(t, bx), &S->q_full, bx * 64,
-                    w.q0 + t * kBM, h, b);
+        tma_load_4d_hint(&p.q_map, smem + L::q(t, bx), &S->q_full, bx * 64,
+                         w.q0 + t * kBM, h, b, once);
   }
   for (int s = 0; s < kMaxSegments; ++s)
     tma_prefetch_desc(kIsK ? &p.k_map[s] : &p.v_map[s]);
@@ -294,9 +298,9 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
     if (!wait_bar(&empty[st], ph ^ 1, S, p.status)) break;
     mbar_arrive_expect_tx(&full[st], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
-      tma_load_4d(kIsK ? &p.k_map[seg] : &p.v_map[seg],
-                  smem + (kIsK ? L::k(st, bx) : L::v(st, bx)), &full[st],
-                  bx * 64, tok0, h, b);
+      tma_load_4d_hint(kIsK ? &p.k_map[seg] : &p.v_map[seg],
+                       smem + (kIsK ? L::k(st, bx) : L::v(st, bx)), &full[st],
+                       bx * 64, tok0, h, b, keep);
     ++issued;
   }
   // Every issued load has landed before the CTA may exit (a no-op wait in

@@ -81,6 +81,34 @@ __device__ __forceinline__ void tma_load_4d(const CUtensorMap* map, void* dst,
       : "memory");
 }
 
+// L2 cache policies for loads: evict_last for tiles that other CTAs read
+// again soon (the streamed K/V of one head), evict_first for tiles read once.
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// tma_load_4d with an L2 cache policy.
+__device__ __forceinline__ void tma_load_4d_hint(const CUtensorMap* map,
+                                                 void* dst, uint64_t* bar,
+                                                 int32_t c0, int32_t c1,
+                                                 int32_t c2, int32_t c3,
+                                                 uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_"
+      "tx::bytes.L2::cache_hint [%0], [%1, {%3, %4, %5, %6}], [%2], %7;" ::"r"(
+          smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_addr(bar)), "r"(c0),
+      "r"(c1), "r"(c2), "r"(c3), "l"(policy)
+      : "memory");
+}
+
 // 4-D tiled store of one box from shared memory (the map's box and swizzle;
 // elements outside the tensor are not written), tracked by bulk groups.
 __device__ __forceinline__ void tma_store_4d(const CUtensorMap* map,
