@@ -36,6 +36,13 @@
 // so this is exact up to rounding.  Before storing P_t(j) the softmax waits
 // until PV_t(j-1) has completed, so O_t is current for the rare rescale.
 //
+// Epilogue: a whole unit's softmax warps stage O_t / l as bf16 in the Q_t
+// buffer (free once every MMA has completed) and one thread per tile writes
+// it with tiled TMA stores; a split unit's key ranges write fp32 partials
+// and the log2-domain LSE for the merge kernel.  The TMA loads carry L2
+// policies: evict_first for the query tiles (one CTA reads them),
+// evict_last for K/V (every unit of the head reads them).
+//
 // Every mbarrier wait is bounded: past the limit the kernel records
 // FASTVR timeout in the control word, all roles stop issuing, in-flight TMA
 // loads and MMAs are drained, TMEM is released and the CTA exits.
