@@ -8,7 +8,8 @@
 //     dV = P^T dO,  dP = dO V^T,  dS = P o (dP - D),
 //     dQ = scale dS K,  dK = scale dS^T Q.
 // Three kernels, no atomics:
-//   delta_kernel  D_i = <dO_i, O_i> (fp32) into the caller's scratch;
+//   delta_kernel  D_i = <dO_i, O_i> (fp32) into the caller's scratch, one
+//                 block per 64 tokens of one (batch, head);
 //   dkdv_kernel   one CTA per 128-key tile: for every query tile that sees it
 //                 S^T = K Q^T and dP^T = V dO^T (SMEM x SMEM -> TMEM); P^T in
 //                 bf16 over S^T (and in registers); dV += P^T dO, then the
@@ -17,11 +18,17 @@
 //                 operand) and the next tile's dP^T;
 //   dq_kernel     one CTA per 128-query tile: for every visible key tile
 //                 S = Q K^T and dP = dO V^T; P in registers (then the next
-//                 tile's S is issued), dS over dP, dQ += dS K.
+//                 tile's S and dP are issued, dP into the other of two
+//                 buffers), dS over dP, dQ += dS K.
 // Visibility is Eq. 1 with window W per (query row, key): a key of chunk c'
 // is seen by queries of chunks c' .. c' + W, a query of chunk c sees keys of
 // chunks c - W .. c; only tiles inside a CTA's visible range are loaded and
-// columns outside each row's range are masked.
+// columns outside each row's range are masked (only tiles that cross a chunk
+// edge take the masked form of the exponential step).
+// CTAs run in head-major order, so the CTAs resident at one time stream the
+// tiles of one or two heads, which stay in L2 (loads carry evict_last for
+// the streamed tiles, evict_first for the resident ones); each CTA writes
+// its output tile through shared memory with tiled TMA stores.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <math.h>
