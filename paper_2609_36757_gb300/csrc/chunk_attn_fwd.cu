@@ -786,14 +786,16 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
 // A CTA merges a block of 32 query rows x 32 columns of one unit: thread
 // (r, g) accumulates columns [4 g, 4 g + 4) of the block for row r, so a
 // warp reads 32 consecutive rows of one column of a part (coalesced).  The
-// parts are walked kPartUnroll at a time with all their loads issued
-// together: the merge reads tens of MB that are mostly still in L2, and it
-// is the latency of those reads, not their volume, that sets its time.  The
-// bf16 rows are written contiguously through shared memory.
+// parts are walked once, kPartUnroll at a time with all their loads issued
+// together, the reference max moving with each group (what was accumulated
+// is rescaled by 2^(m_old - m_new)): the merge reads tens of MB that are
+// mostly still in L2, and it is the latency of those reads, not their
+// volume, that sets its time.  The bf16 rows are written contiguously
+// through shared memory.
 constexpr int kMergeRows = 32;
 constexpr int kMergeCols = 32;
 constexpr int kMergeThreads = kMergeRows * kMergeCols / 4;  // 256
-constexpr int kPartUnroll = 8;
+constexpr int kPartUnroll = 16;
 
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads)
@@ -817,15 +819,7 @@ combine_kernel(const __grid_constant__ TcParams p) {
   // every part this block reads lies in the workspace
   if (!in_bounds(k0 + p.split - 1, p.ws_parts, p.status)) return;
   const float* lse = p.ws_lse + (size_t)k0 * kUnitRows + r_unit;
-  float m = -INFINITY;
-  for (int i0 = 0; i0 < p.split; i0 += kPartUnroll) {
-    float l8[kPartUnroll];
-#pragma unroll
-    for (int u = 0; u < kPartUnroll; ++u)
-      l8[u] = i0 + u < p.split ? lse[(size_t)(i0 + u) * kUnitRows] : -INFINITY;
-#pragma unroll
-    for (int u = 0; u < kPartUnroll; ++u) m = fmaxf(m, l8[u]);
-  }
+  float m = -INFINITY;  // reference: the max of the parts seen so far
   float acc[kCols];
 #pragma unroll
   for (int x = 0; x < kCols; ++x) acc[x] = 0.f;
@@ -842,6 +836,16 @@ combine_kernel(const __grid_constant__ TcParams p) {
       for (int x = 0; x < kCols; ++x)
         v[u][x] = have ? src[(size_t)x * kUnitRows] : 0.f;
     }
+    float mg = m;
+#pragma unroll
+    for (int u = 0; u < kPartUnroll; ++u) mg = fmaxf(mg, w8[u]);
+    if (mg == -INFINITY) continue;  // nothing finite yet
+    // 0 on the first finite group (nothing accumulated), else <= 1
+    const float sc = m == -INFINITY ? 0.f : ex2(m - mg);
+    wsum *= sc;
+#pragma unroll
+    for (int x = 0; x < kCols; ++x) acc[x] *= sc;
+    m = mg;
 #pragma unroll
     for (int u = 0; u < kPartUnroll; ++u) {
       const float wi = ex2(w8[u] - m);  // 0 for the missing parts
