@@ -51,7 +51,29 @@ CASES = [
 ]
 
 
-@pytest.mark.parametrize("w", CASES, ids=lambda w: w.name)
+def _random_cases(n: int, seed: int):
+    """Seeded random one-shot shapes (head dim, frame size, chunk size,
+    window, ragged last chunk), at most ~2300 tokens so that the oracle's
+    float64 backward stays quick."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for i in range(n):
+        k = int(rng.integers(1, 4))
+        out.append(WL.custom(
+            f"rand{i}", batch=int(rng.integers(1, 3)),
+            heads=int(rng.integers(1, 3)),
+            head_dim=int(rng.choice([64, 128])),
+            tokens_per_frame=int(rng.integers(1, 151)),
+            frames_per_chunk=k, num_chunks=int(rng.integers(2, 6)),
+            window_chunks=int(rng.choice([-1, 0, 1, 2])),
+            last_chunk_frames=int(rng.integers(0, k)), seed=400 + i))
+    return out
+
+
+RANDOM = _random_cases(6, 3607)
+
+
+@pytest.mark.parametrize("w", CASES + RANDOM, ids=lambda w: w.name)
 def test_backward_vs_oracle(w):
     from paper_2609_36757_gb300 import fastvr as FV
     qs, ks, vs = [], [], []

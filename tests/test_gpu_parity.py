@@ -85,6 +85,35 @@ def test_small_stream_every_element(w):
     err.check()
 
 
+def _random_streams(n: int, seed: int):
+    """Seeded random small streams: head dim, frame size (ragged against the
+    128-row tiles, down to one token), chunk size, window and a ragged last
+    chunk drawn at random; small enough for the oracle to check every
+    element."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for i in range(n):
+        k = int(rng.integers(1, 4))
+        out.append(WL.custom(
+            f"rand{i}", batch=int(rng.integers(1, 3)),
+            heads=int(rng.integers(1, 4)),
+            head_dim=int(rng.choice([64, 128])),
+            tokens_per_frame=int(rng.integers(1, 260)),
+            frames_per_chunk=k, num_chunks=int(rng.integers(2, 6)),
+            window_chunks=int(rng.choice([-1, 0, 1, 2])),
+            last_chunk_frames=int(rng.integers(0, k)), seed=300 + i))
+    return out
+
+
+RANDOM = _random_streams(12, 2609)
+
+
+@pytest.mark.parametrize("w", RANDOM, ids=lambda w: w.name)
+def test_random_small_stream_every_element(w):
+    err = run_stream(w)
+    err.check()
+
+
 @pytest.mark.parametrize("w", SMALL[:3], ids=lambda w: w.name)
 def test_streamed_gpu_equals_oneshot_oracle(FV, w):
     att = FV.StreamingAttention(FV.config_from_workload(w))
