@@ -113,6 +113,7 @@ struct TcParams {
   // fastest; the first units_full run whole, the rest are cut into `split`
   // key-tile ranges whose partial results go to the workspace.
   int32_t q_pairs, units_full, split;
+  int32_t sms;  // SM count: CTA index / sms is a CTA's wave
   float* ws;      // partial O: [part][d][kUnitRows]
   float* ws_lse;  // partial log2-domain LSE: [part][kUnitRows]
   int32_t ws_parts;  // partial results the workspace holds
@@ -129,7 +130,18 @@ struct Work {
   int nqt;     // query tiles with at least one row in the chunk (1 or 2)
   int part;    // -1: whole unit, final output; else workspace slot
   int kv0, kv1;  // one-shot: the unit's key token range [kv0, kv1)
+  bool rev;    // walk the key tiles last to first
 };
+
+// Whole units in odd waves (CTA index / SM count) walk their key tiles last
+// to first.  Consecutive units of a head run together, so a head whose units
+// straddle two waves is streamed by the second wave right after the first:
+// walking back, that wave starts on the tiles the first one loaded last,
+// which are still in L2, instead of on the oldest ones.  The online softmax
+// does not depend on the order (up to rounding).
+__device__ __forceinline__ bool odd_wave(const TcParams& p) {
+  return ((int)blockIdx.x / p.sms) & 1;
+}
 
 // One-shot launches: the query pairs are grouped from the end of the
 // sequence into blocks of kOneShotBlock pairs; unit x takes block
@@ -161,6 +173,7 @@ __device__ __forceinline__ Work oneshot_work(const TcParams& p) {
   w.j0 = 0;
   w.n = (w.kv1 - w.kv0 + kBN - 1) / kBN;
   w.part = -1;
+  w.rev = odd_wave(p);
   return w;
 }
 
@@ -187,6 +200,7 @@ __device__ __forceinline__ Work cta_work(const TcParams& p) {
   w.j0 = (int)((int64_t)idx * p.total_tiles / nparts);
   w.n = (int)((int64_t)(idx + 1) * p.total_tiles / nparts) - w.j0;
   w.part = part;
+  w.rev = part < 0 && odd_wave(p);
   return w;
 }
 
@@ -298,10 +312,11 @@ __device__ void producer(const TcParams& p, uint8_t* smem, Shared* S,
     const int st = j % kStages;
     const uint32_t ph = (j / kStages) & 1;
     int seg, tok0, valid;
+    const int jt = w.rev ? w.n - 1 - j : j;
     if (kOneShot)
-      oneshot_tile(w.kv0, w.kv1, j, seg, tok0, valid);
+      oneshot_tile(w.kv0, w.kv1, jt, seg, tok0, valid);
     else
-      tile_coord(p, w.j0 + j, seg, tok0, valid);
+      tile_coord(p, w.j0 + jt, seg, tok0, valid);
     if (!wait_bar(&empty[st], ph ^ 1, S, p.status)) break;
     mbar_arrive_expect_tx(&full[st], L::kNB * kBox);
     for (int bx = 0; bx < L::kNB; ++bx)
@@ -595,7 +610,7 @@ __device__ __forceinline__ void mask_range_max32(uint32_t (&sc)[32], int c,
 template <int D, bool kOneShot>
 __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
                              int t, int nqt, int wq, int lane, int j0, int n,
-                             int kv0, int kv1, int q0) {
+                             int kv0, int kv1, int q0, bool rev) {
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
   const uint32_t tS = tmem + kTmemS + lane_off;
   const uint32_t tP = tmem + kTmemP + t * 64 + lane_off;
@@ -618,10 +633,11 @@ __device__ void softmax_role(const TcParams& p, Shared* S, uint32_t tmem,
   }
   for (int j = 0; j < n; ++j) {
     int seg, tok0, valid;
+    const int jt = rev ? n - 1 - j : j;  // the producers' order
     if (kOneShot)
-      oneshot_tile(kv0, kv1, j, seg, tok0, valid);
+      oneshot_tile(kv0, kv1, jt, seg, tok0, valid);
     else
-      tile_coord(p, j0 + j, seg, tok0, valid);
+      tile_coord(p, j0 + jt, seg, tok0, valid);
     if (!(ok = wait_bar(&S->s_full[t], j & 1, S, p.status))) break;
     tc_fence_after();
     uint32_t s[4][32];
@@ -938,7 +954,7 @@ chunk_attn_tc_kernel(const __grid_constant__ TcParams p) {
     // A query tile that lies past the end of the chunk has no work.
     if (warp / 4 < w.nqt)
       softmax_role<D, kOneShot>(p, S, tmem, warp / 4, w.nqt, warp % 4, lane,
-                                w.j0, w.n, w.kv0, w.kv1, w.q0);
+                                w.j0, w.n, w.kv0, w.kv1, w.q0, w.rev);
   }
   tc_fence_before();
   __syncthreads();
@@ -1046,7 +1062,8 @@ cudaError_t launch_d(const AttnParams& a, cudaStream_t stream, int* launches) {
 
   p.q_pairs = (a.q_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);
   const int units = p.q_pairs * a.heads * a.batch;
-  split_units(units, tiles, sm_count(), a.workspace_parts, &p.units_full,
+  p.sms = sm_count();
+  split_units(units, tiles, p.sms, a.workspace_parts, &p.units_full,
               &p.split);
   p.ws_lse = p.ws + (size_t)a.workspace_parts * D * kUnitRows;
   const int grid = p.units_full + (units - p.units_full) * p.split;
@@ -1107,6 +1124,7 @@ cudaError_t launch_oneshot_d(const OneShotParams& a, cudaStream_t stream) {
   p.window = a.window;
   p.q_pairs = (a.seq_tokens + kQTiles * kBM - 1) / (kQTiles * kBM);
   p.split = 1;
+  p.sms = sm_count();
   const int grid = p.q_pairs * a.heads * a.batch;
   p.units_full = grid;
   const int smem = Layout<D>::bytes;
