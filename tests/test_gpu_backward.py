@@ -106,3 +106,34 @@ def test_backward_is_deterministic():
     b = FV.blockcausal_attention_bwd(cfg, q, k, v, o, do, lse)
     for x, y in zip(a, b):
         assert torch.equal(x, y)
+
+
+def test_backward_train_clip_full_heads_vs_oracle():
+    """The training clip that the bench times (train-1024-clip: 12 frames x
+    1024 tokens, k = 3, W = 1, 24 heads, d = 128), run whole on the GPU; the
+    first and the last head compared in full with the oracle's float64
+    backward (the oracle works per (batch, head), so a head is an exact
+    sub-problem; a few seconds of BLAS per head for its 12288 x 12288
+    matrices on the GPU host)."""
+    from paper_2609_36757_gb300 import fastvr as FV
+    w = WL.TRAIN_CLIP
+    qs, ks, vs = [], [], []
+    for _, q, k, v in WL.chunk_stream(w):
+        qs.append(q), ks.append(k), vs.append(v)
+    q, k, v = torch.cat(qs, 1), torch.cat(ks, 1), torch.cat(vs, 1)
+    g = torch.Generator().manual_seed(w.seed + 1000)
+    do = torch.randn(q.shape, generator=g).to(torch.bfloat16)
+    cfg = FV.config_from_workload(w)
+    qd, kd, vd, dod = q.cuda(), k.cuda(), v.cuda(), do.cuda()
+    o, lse = FV.blockcausal_attention(cfg, qd, kd, vd, want_lse=True)
+    dq, dk, dv = FV.blockcausal_attention_bwd(cfg, qd, kd, vd, o, dod, lse)
+    torch.cuda.synchronize()
+    dq, dk, dv = dq.cpu(), dk.cpu(), dv.cpu()
+    for h in (0, w.heads - 1):
+        sl = slice(h, h + 1)
+        ref = OA.blockcausal_attention_bwd(
+            to64(q[:, :, sl]), to64(k[:, :, sl]), to64(v[:, :, sl]),
+            to64(do[:, :, sl]), w.tokens_per_frame, w.frames_per_chunk,
+            w.window_chunks, w.softmax_scale)
+        for name, got, r in zip(("dq", "dk", "dv"), (dq, dk, dv), ref):
+            _check(got[:, :, sl], r, f"{name} head {h}")
